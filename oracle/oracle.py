@@ -1,0 +1,467 @@
+"""CPU oracle for provenance-bound KV-cache keys -- TEST INFRASTRUCTURE.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline / reference leg
+of ``bench.py`` may import this module.  It shares no code with the CUDA path
+(``paper_2609_38706_gb300``) and imports nothing from it.
+
+Every function restates one passage of the paper ("Preserving Provenance in
+Shared KV Caches for LLM Serving") or one of the stated readings where the
+paper is silent:
+
+* ``canonicalize``   -- Sec. 5.3 "Worker-level digest": bind resolved values,
+  never a launch string such as ``auto``; identity functions must be injective
+  and cross-worker stable (Sec. 5.1).  The synonym table is a reading.
+* ``enc``            -- Sec. 5.2, Eq. 3: an injective, length-prefixed encoder.
+  Byte layout is a reading: LE32(field count) then LE32(len) || bytes per field.
+* ``descriptor_digest`` -- d = H(enc(...)) of Eq. 3 with H = SHA-256.
+* ``chunk_digest`` / ``chain_step`` / ``derive_keys`` -- the connector key f of
+  Eq. 3 instantiated as c_i = SHA-256(LE int32 tokens of chunk i) and
+  k_i = SHA-256(k_{i-1} || d || c_i) with k_{-1} = 0^32, full chunks only
+  (Sec. 4.4: prefixes below one chunk never collide).  Computed by the plain C
+  library ``pk_oracle.c`` (FIPS 180-4 written out).
+* ``DictTable``      -- the shared store of Sec. 2.1 reduced to a map from the
+  128-bit key prefix (Sec. 5.3, "the encoding keeps 128 bits") to a chunk
+  slot.  Lookup returns the longest all-hit prefix (Sec. 2.1: on a local miss
+  the connector queries the store; a hit skips that prefill, a miss computes
+  and writes new state).  Store inserts in array order, the first occurrence
+  wins, an existing key keeps its slot.
+* ``SortedTable``    -- the same semantics computed with sort / searchsorted so
+  that million-entry tables stay tractable; checked against ``DictTable``.
+
+Pins live in ``tests/test_oracle_*.py``: SHA-256 against hashlib and the
+FIPS 180-2 Appendix B digests, ``enc`` injectivity by property tests, the key
+chain against the contract invariants Eq. 1, Eq. 2 and Eq. 4 by brute force,
+and the tables against each other and against closed-form counts.  Parity
+unpinned by the paper (stated conventions only): the field order of ``enc``,
+its byte layout, the chain's operand order and zero seed, the partial-chunk
+rule, which 16 bytes form the prefix, and the canonical synonym spellings.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+from typing import Iterable, Mapping, Sequence
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "pk_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "_build", "libpk_oracle.so")
+
+# Status vocabulary (the C-ABI's published codes, restated here as plain data).
+PK_OK = 0
+PK_ERR_ARG = -1
+PK_ERR_CAPACITY = -2
+PK_ERR_UNRESOLVED = -3
+PK_ERR_FIELD_TOO_LONG = -4
+PK_ERR_TABLE_FULL = -5
+PK_ERR_PROBE_LIMIT = -6
+PK_ERR_RESERVED_KEY = -7
+
+STORE_SKIPPED = 0
+STORE_INSERTED = 1
+STORE_PRESENT = 2
+NO_SLOT = 0xFFFFFFFF
+
+MAX_FIELD_BYTES = 4096
+
+# Registry v1 (Sec. 5.1 dimensions plus the model identity the connector already
+# carries, Sec. 5.3).  Order is a stated convention.
+REGISTRY_V1 = ("model_id", "weight_precision", "weight_version", "adapter_id", "kv_format", "salt")
+_RESOLVED_FIELDS = ("weight_precision", "kv_format")
+_SYNONYMS = {
+    "bfloat16": "bf16",
+    "float16": "fp16",
+    "half": "fp16",
+    "float32": "fp32",
+    "float": "fp32",
+    "float8_e4m3fn": "fp8_e4m3",
+    "float8_e5m2": "fp8_e5m2",
+}
+
+
+class OracleError(Exception):
+    def __init__(self, code: int, msg: str = ""):
+        super().__init__(f"{code}: {msg}")
+        self.code = code
+
+
+# --------------------------------------------------------------------------
+# C library
+# --------------------------------------------------------------------------
+_lib = None
+_lib_lock = threading.Lock()
+
+
+def build(force: bool = False) -> str:
+    """Compile pk_oracle.c with gcc into oracle/_build/libpk_oracle.so."""
+    os.makedirs(os.path.dirname(_LIB_PATH), exist_ok=True)
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-o", tmp, _SRC])
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def lib():
+    global _lib
+    with _lib_lock:
+        if _lib is None:
+            build()
+            L = ctypes.CDLL(_LIB_PATH)
+            u8p = ctypes.POINTER(ctypes.c_uint8)
+            L.oracle_sha256.argtypes = [ctypes.c_void_p, ctypes.c_uint64, ctypes.c_void_p]
+            L.oracle_sha256.restype = None
+            L.oracle_chunk_digest.argtypes = [ctypes.c_void_p, ctypes.c_uint32, ctypes.c_void_p]
+            L.oracle_chunk_digest.restype = None
+            L.oracle_chain_step.argtypes = [ctypes.c_void_p] * 4
+            L.oracle_chain_step.restype = None
+            L.oracle_request_keys.argtypes = [ctypes.c_void_p, ctypes.c_uint64, ctypes.c_uint32,
+                                              ctypes.c_void_p, ctypes.c_void_p]
+            L.oracle_request_keys.restype = ctypes.c_uint64
+            L.oracle_derive_keys.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_uint32,
+                                             ctypes.c_uint32, ctypes.c_void_p, ctypes.c_void_p,
+                                             ctypes.c_uint32, ctypes.c_void_p, ctypes.c_void_p]
+            L.oracle_derive_keys.restype = ctypes.c_int64
+            L.oracle_max_threads.argtypes = []
+            L.oracle_max_threads.restype = ctypes.c_int
+            L.oracle_set_threads.argtypes = [ctypes.c_int]
+            L.oracle_set_threads.restype = None
+            L.oracle_constants.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+            L.oracle_constants.restype = None
+            del u8p
+            _lib = L
+    return _lib
+
+
+def _ptr(a: np.ndarray) -> int:
+    return a.ctypes.data
+
+
+def max_threads() -> int:
+    return int(lib().oracle_max_threads())
+
+
+def set_threads(n: int) -> None:
+    lib().oracle_set_threads(int(n))
+
+
+def constants() -> tuple[np.ndarray, np.ndarray]:
+    k = np.zeros(64, np.uint32)
+    h = np.zeros(8, np.uint32)
+    lib().oracle_constants(_ptr(k), _ptr(h))
+    return k, h
+
+
+# --------------------------------------------------------------------------
+# SHA-256 and the key chain
+# --------------------------------------------------------------------------
+def sha256(msg: bytes) -> bytes:
+    buf = np.frombuffer(bytes(msg) + b"\0", dtype=np.uint8)
+    out = np.zeros(32, np.uint8)
+    lib().oracle_sha256(_ptr(buf), len(msg), _ptr(out))
+    return out.tobytes()
+
+
+def chunk_digest(tokens: np.ndarray) -> bytes:
+    """c = SHA-256(little-endian int32 serialisation of the chunk's tokens)."""
+    t = np.ascontiguousarray(tokens, dtype=np.int32)
+    out = np.zeros(32, np.uint8)
+    lib().oracle_chunk_digest(_ptr(t) if t.size else 0, t.size, _ptr(out))
+    return out.tobytes()
+
+
+def chain_step(prev: bytes, d: bytes, c: bytes) -> bytes:
+    """k_i = SHA-256(k_{i-1} || d || c_i)."""
+    a = [np.frombuffer(x, np.uint8).copy() for x in (prev, d, c)]
+    assert all(x.size == 32 for x in a)
+    out = np.zeros(32, np.uint8)
+    lib().oracle_chain_step(_ptr(a[0]), _ptr(a[1]), _ptr(a[2]), _ptr(out))
+    return out.tobytes()
+
+
+def request_keys(tokens: np.ndarray, C: int, d: bytes) -> np.ndarray:
+    """Keys of one request: uint8[floor(T/C), 32]."""
+    t = np.ascontiguousarray(tokens, dtype=np.int32)
+    n = t.size // C
+    out = np.zeros((max(n, 1), 32), np.uint8)
+    dd = np.frombuffer(d, np.uint8).copy()
+    got = lib().oracle_request_keys(_ptr(t) if t.size else 0, t.size, C, _ptr(dd), _ptr(out))
+    assert got == n
+    return out[:n]
+
+
+def derive_keys(tokens: np.ndarray, tok_off: np.ndarray, C: int, desc_idx: np.ndarray,
+                digests: np.ndarray) -> tuple[np.ndarray, np.ndarray]:
+    """All keys of a batch -> (key_off int64[R+1], keys uint8[N, 32])."""
+    tokens = np.ascontiguousarray(tokens, dtype=np.int32)
+    tok_off = np.ascontiguousarray(tok_off, dtype=np.int64)
+    desc_idx = np.ascontiguousarray(desc_idx, dtype=np.uint32)
+    digests = np.ascontiguousarray(digests, dtype=np.uint8).reshape(-1, 32)
+    R = tok_off.size - 1
+    if C <= 0:
+        raise OracleError(PK_ERR_ARG, "chunk size must be positive")
+    lens = np.diff(tok_off)
+    N = int((lens // C).sum()) if R > 0 else 0
+    key_off = np.zeros(R + 1, np.int64)
+    keys = np.zeros((max(N, 1), 32), np.uint8)
+    got = lib().oracle_derive_keys(_ptr(tokens) if tokens.size else 0, _ptr(tok_off), R, C,
+                                   _ptr(desc_idx) if R else 0, _ptr(digests) if digests.size else 0,
+                                   digests.shape[0], _ptr(key_off), _ptr(keys))
+    if got < 0:
+        raise OracleError(PK_ERR_ARG, "bad offsets or descriptor index")
+    assert got == N
+    return key_off, keys[:N]
+
+
+# --------------------------------------------------------------------------
+# Descriptor canonicalisation and enc (Sec. 5.2, 5.3)
+# --------------------------------------------------------------------------
+def _as_bytes(v) -> bytes:
+    if v is None:
+        return b""
+    if isinstance(v, str):
+        return v.encode("utf-8")
+    return bytes(v)
+
+
+def _ascii_lower(b: bytes) -> bytes:
+    return bytes(c + 32 if 65 <= c <= 90 else c for c in b)
+
+
+def canonicalize(desc: Mapping) -> tuple[bytes, ...]:
+    """Resolved, injective identities for registry v1 (+ appended extra fields).
+
+    ``desc`` maps the six registry names to str/bytes (absent == empty) and may
+    carry ``extra``: a sequence of appended field values (Prop. 1).
+    """
+    fields = []
+    for name in REGISTRY_V1:
+        v = _as_bytes(desc.get(name, b""))
+        if name in _RESOLVED_FIELDS:
+            v = _ascii_lower(v)
+            s = v.decode("latin-1")
+            v = _SYNONYMS.get(s, s).encode("latin-1")
+            if v == b"" or v == b"auto":
+                raise OracleError(PK_ERR_UNRESOLVED, f"{name} must be a resolved value")
+        if len(v) > MAX_FIELD_BYTES:
+            raise OracleError(PK_ERR_FIELD_TOO_LONG, name)
+        fields.append(v)
+    for v in desc.get("extra", ()) or ():
+        v = _as_bytes(v)
+        if len(v) > MAX_FIELD_BYTES:
+            raise OracleError(PK_ERR_FIELD_TOO_LONG, "extra")
+        fields.append(v)
+    return tuple(fields)
+
+
+def enc(fields: Sequence[bytes]) -> bytes:
+    """LE32(number of fields) || for each field: LE32(length) || bytes."""
+    out = bytearray(len(fields).to_bytes(4, "little"))
+    for f in fields:
+        f = bytes(f)
+        out += len(f).to_bytes(4, "little")
+        out += f
+    return bytes(out)
+
+
+def descriptor_digest(desc: Mapping) -> bytes:
+    """d = SHA-256(enc(canonicalize(desc)))."""
+    return sha256(enc(canonicalize(desc)))
+
+
+def descriptor_digests(descs: Iterable[Mapping]) -> np.ndarray:
+    ds = [descriptor_digest(d) for d in descs]
+    if not ds:
+        return np.zeros((0, 32), np.uint8)
+    return np.frombuffer(b"".join(ds), np.uint8).reshape(-1, 32).copy()
+
+
+# --------------------------------------------------------------------------
+# Table semantics
+# --------------------------------------------------------------------------
+def prefix128(keys: np.ndarray) -> np.ndarray:
+    """First 16 bytes of each key (standard digest byte order)."""
+    keys = np.ascontiguousarray(keys, dtype=np.uint8)
+    return np.ascontiguousarray(keys.reshape(-1, keys.shape[-1])[:, :16])
+
+
+class DictTable:
+    """Exact-match map from 16-byte key prefixes to uint32 slots.
+
+    Capacity rule: at most ``capacity - 1`` entries (one slot always stays
+    empty); an insertion that would exceed it is refused with TABLE_FULL.
+    The all-zero prefix is the empty marker and cannot be stored.
+    """
+
+    def __init__(self, capacity: int):
+        if capacity < 2 or capacity & (capacity - 1):
+            raise OracleError(PK_ERR_CAPACITY, "capacity must be a power of two >= 2")
+        self.capacity = capacity
+        self.map: dict[bytes, int] = {}
+
+    def __len__(self):
+        return len(self.map)
+
+    def store(self, keys: np.ndarray, slots: np.ndarray):
+        """Insert in array order -> (result int32[n], slot_out uint32[n])."""
+        p = prefix128(keys)
+        slots = np.asarray(slots, dtype=np.uint32)
+        n = p.shape[0]
+        result = np.zeros(n, np.int32)
+        slot_out = np.full(n, NO_SLOT, np.uint32)
+        zero = bytes(16)
+        for i in range(n):
+            k = p[i].tobytes()
+            if k == zero:
+                result[i] = PK_ERR_RESERVED_KEY
+                continue
+            if int(slots[i]) == NO_SLOT:
+                result[i] = PK_ERR_ARG
+                continue
+            if k in self.map:
+                result[i] = STORE_PRESENT
+                slot_out[i] = self.map[k]
+            elif len(self.map) + 1 >= self.capacity:
+                result[i] = PK_ERR_TABLE_FULL
+            else:
+                self.map[k] = int(slots[i])
+                result[i] = STORE_INSERTED
+                slot_out[i] = int(slots[i])
+        return result, slot_out
+
+    def get(self, keys: np.ndarray) -> np.ndarray:
+        p = prefix128(keys)
+        return np.array([self.map.get(p[i].tobytes(), NO_SLOT) for i in range(p.shape[0])],
+                        dtype=np.uint32)
+
+
+class SortedTable:
+    """Same semantics as DictTable, computed with sort / searchsorted.
+
+    Holds unique prefixes sorted bytewise with the slot of each one's first
+    insertion.  Used for tables of millions of entries.
+    """
+
+    def __init__(self, capacity: int):
+        if capacity < 2 or capacity & (capacity - 1):
+            raise OracleError(PK_ERR_CAPACITY, "capacity must be a power of two >= 2")
+        self.capacity = capacity
+        self.keys = np.zeros(0, dtype="V16")
+        self.slots = np.zeros(0, np.uint32)
+
+    def __len__(self):
+        return int(self.keys.size)
+
+    @staticmethod
+    def _v16(keys: np.ndarray) -> np.ndarray:
+        return prefix128(keys).view("V16").reshape(-1)
+
+    def _find(self, q: np.ndarray) -> tuple[np.ndarray, np.ndarray]:
+        if self.keys.size == 0:
+            return np.zeros(q.size, bool), np.zeros(q.size, np.int64)
+        pos = np.searchsorted(self.keys, q)
+        posc = np.minimum(pos, self.keys.size - 1)
+        found = self.keys[posc] == q
+        return found, posc
+
+    def get(self, keys: np.ndarray) -> np.ndarray:
+        q = self._v16(keys)
+        found, pos = self._find(q)
+        out = np.full(q.size, NO_SLOT, np.uint32)
+        out[found] = self.slots[pos[found]]
+        return out
+
+    def store(self, keys: np.ndarray, slots: np.ndarray):
+        q = self._v16(keys)
+        slots = np.asarray(slots, dtype=np.uint32)
+        n = q.size
+        result = np.zeros(n, np.int32)
+        slot_out = np.full(n, NO_SLOT, np.uint32)
+        zero = np.zeros(1, dtype="V16")[0]
+        bad_key = q == zero
+        bad_slot = slots == NO_SLOT
+        result[bad_key] = PK_ERR_RESERVED_KEY
+        result[bad_slot & ~bad_key] = PK_ERR_ARG
+        ok = ~(bad_key | bad_slot)
+        found, pos = self._find(q)
+        pre = ok & found
+        result[pre] = STORE_PRESENT
+        slot_out[pre] = self.slots[pos[pre]]
+        new = np.nonzero(ok & ~found)[0]
+        if new.size:
+            uq, first, inv = np.unique(q[new], return_index=True, return_inverse=True)
+            # insertion order of the new distinct keys = order of first occurrence
+            order = np.argsort(first, kind="stable")
+            room = max(self.capacity - 1 - len(self), 0)
+            accepted_rank = np.zeros(uq.size, bool)
+            accepted_rank[order[:room]] = True
+            win_idx = new[first]                       # batch index of each distinct key's first occurrence
+            acc = accepted_rank[inv]
+            idx_acc = new[acc]
+            is_first = idx_acc == win_idx[inv[acc]]
+            result[idx_acc[is_first]] = STORE_INSERTED
+            result[idx_acc[~is_first]] = STORE_PRESENT
+            slot_out[idx_acc] = slots[win_idx[inv[acc]]]
+            result[new[~acc]] = PK_ERR_TABLE_FULL
+            ins_keys = uq[accepted_rank]
+            ins_slots = slots[win_idx[accepted_rank]]
+            allk = np.concatenate([self.keys, ins_keys])
+            alls = np.concatenate([self.slots, ins_slots])
+            o = np.argsort(allk, kind="stable")
+            self.keys, self.slots = allk[o], alls[o]
+        return result, slot_out
+
+
+def lookup(table, keys: np.ndarray, key_off: np.ndarray):
+    """Probe every key -> (hit_chunks int32[R], slots uint32[N]).
+
+    hit_chunks[r] = h_r, the largest j such that chunks 0..j-1 of request r are
+    all present; slots[i] is the stored slot of key i or NO_SLOT.
+    """
+    key_off = np.asarray(key_off, dtype=np.int64)
+    R = key_off.size - 1
+    slots = table.get(keys) if keys.shape[0] else np.zeros(0, np.uint32)
+    hit = np.zeros(R, np.int32)
+    for r in range(R):
+        s = slots[key_off[r]:key_off[r + 1]]
+        miss = np.nonzero(s == NO_SLOT)[0]
+        hit[r] = int(miss[0]) if miss.size else s.size
+    return hit, slots
+
+
+def store_misses(table, keys: np.ndarray, key_off: np.ndarray, hit_chunks: np.ndarray,
+                 slots: np.ndarray):
+    """Store the keys of every miss range [h_r, n_r), in global key order.
+
+    Returns (result int32[N], slot_out uint32[N]); entries below h_r are SKIPPED.
+    """
+    key_off = np.asarray(key_off, dtype=np.int64)
+    N = keys.shape[0]
+    idx = []
+    for r in range(key_off.size - 1):
+        idx.extend(range(int(key_off[r]) + int(hit_chunks[r]), int(key_off[r + 1])))
+    idx = np.asarray(idx, dtype=np.int64)
+    result = np.full(N, STORE_SKIPPED, np.int32)
+    slot_out = np.full(N, NO_SLOT, np.uint32)
+    if idx.size:
+        res, so = table.store(keys[idx], np.asarray(slots, np.uint32)[idx])
+        result[idx] = res
+        slot_out[idx] = so
+    return result, slot_out
+
+
+def seed_table(table, seed_keys: np.ndarray, filler: np.ndarray, target_entries: int):
+    """Pre-fill a table: the seed keys in order (slot = list index), then filler
+    keys, continuing the index, until it holds ``target_entries`` entries."""
+    n_seed = seed_keys.shape[0]
+    if n_seed:
+        table.store(seed_keys, np.arange(n_seed, dtype=np.uint32))
+    need = target_entries - len(table)
+    if need > 0:
+        if need > filler.shape[0]:
+            raise OracleError(PK_ERR_ARG, "not enough filler keys")
+        table.store(filler[:need], np.arange(n_seed, n_seed + need, dtype=np.uint32))
+    return table
