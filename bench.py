@@ -1,0 +1,397 @@
+#!/usr/bin/env python3
+"""Benchmark: provenance-bound key derivation + longest-prefix lookup + store
+of the misses on one GB300, through the libpk C-ABI.
+
+One step = one pass of the whole hot path over one batch:
+  a0  canonicalise + encode the batch's descriptors (host), SHA-256 -> d (device)
+  a1  chunk digests c_i          a2  chained keys k_i
+  a3  probe every key            a4  store the miss ranges
+Default workload: the multi-adapter serving configuration (1024 requests x
+4096 tokens, chunk 256, 32 descriptors, table of 2^20 entries at load 0.5).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the CPU oracle on the same workload
+
+Timing: each step is bracketed by CUDA events on the launching stream; before
+each step the table is restored to its seeded state (pk_table_load) and L2 is
+flushed by writing a 256 MiB buffer, both outside the events.  A spin kernel
+queued ahead of each step keeps the device busy while the host enqueues it,
+so the events see device time only (`value`).  The `e2e` figure instead
+starts on an idle stream and includes the host-to-device copy of the batch's
+inputs from pinned memory, the host canonicalisation and every launch, and
+the device-to-host copy of the results.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "tokens keyed+looked up/sec and % of SHA-256/HBM roofline (1 GB300)"
+SHA_OPS_PER_COMPRESSION = 1384      # 64 rounds x 14 + 48 schedule words x 10 + 8 feed-forward
+SMS, LANES_PER_SM = 152, 128        # 4 SM sub-partitions x 32 lanes, one instruction each per clock
+L2_FLUSH_BYTES = 256 << 20
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "sm_max_mhz": d.get("sm_max_mhz", 2070.0), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "sm_max_mhz": 2070.0, "source": "fallback"}
+
+
+def compressions(n_keys: int, C: int) -> tuple[int, int]:
+    """SHA-256 compressions per batch: chunk digests (ceil((4C + 9) / 64) each)
+    and chain steps (a 96-byte message = 2 each)."""
+    per_chunk = (4 * C + 9 + 63) // 64
+    return n_keys * per_chunk, 2 * n_keys
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"pk_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        self.proc.wait()
+        self.f.close()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for name, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(name)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def cpu_oracle_pass(wl, d_ref, table, snapshot_keys):
+    """One step of the oracle on a whole batch: keys, lookup, store of the
+    misses; then the inserted keys are removed again so that every pass sees
+    the same table."""
+    import oracle as O
+    b = wl.batch
+    ko, keys = O.derive_keys(b.tokens, b.tok_off, wl.chunk_tokens, b.desc_idx, d_ref)
+    hit, slots = O.lookup(table, keys, ko)
+    new_slots = np.arange(keys.shape[0], dtype=np.uint32) + (1 << 30)
+    res, _ = O.store_misses(table, keys, ko, hit, new_slots)
+    for i in np.nonzero(res == O.STORE_INSERTED)[0]:
+        del table.map[O.prefix128(keys[i:i + 1])[0].tobytes()]
+    assert len(table) == snapshot_keys
+    return keys.shape[0]
+
+
+def oracle_setup(wl):
+    import oracle as O
+    from paper_2609_38706_gb300 import workloads as W
+    d_ref = O.descriptor_digests(wl.descriptors)
+    pko, pkeys = O.derive_keys(wl.prior.tokens, wl.prior.tok_off, wl.chunk_tokens, wl.prior.desc_idx, d_ref)
+    table = O.seed_table(O.DictTable(wl.capacity), W.seed_list(pkeys, pko, wl.prior_chunks), wl.filler,
+                         wl.target_entries)
+    return d_ref, table
+
+
+def run_cpu_baseline(wl, seconds: float) -> dict:
+    import oracle as O
+    d_ref, table = oracle_setup(wl)
+    n0 = len(table)
+    passes, t0 = 0, time.perf_counter()
+    while True:
+        cpu_oracle_pass(wl, d_ref, table, n0)
+        passes += 1
+        el = time.perf_counter() - t0
+        if el >= seconds or passes >= 1000:
+            break
+    return {"value": wl.tokens_keyed() * passes / el, "unit": "tokens/s", "cores": O.max_threads(),
+            "kind": "oracle",
+            "sample": f"{passes} full passes of the {wl.name} batch ({wl.batch.R} requests) in {el:.1f} s: "
+                      "C FIPS 180-4 SHA-256 (OpenMP over requests) + Python dict table"}
+
+
+def workload_config(wl, args) -> dict:
+    lens = np.diff(wl.batch.tok_off)
+    return {"workload": f"{wl.name}: {wl.batch.R} requests x {int(lens.max()) if lens.size else 0} tokens, "
+                        f"chunk {wl.chunk_tokens}, {len(wl.descriptors)} descriptors, table 2^{wl.capacity_log2} "
+                        f"slots seeded to {wl.target_entries} entries",
+            "requests": wl.batch.R, "tokens": wl.batch.n_tokens, "chunk_tokens": wl.chunk_tokens,
+            "keys_per_step": wl.n_keys(), "descriptors": len(wl.descriptors), "table_slots": wl.capacity,
+            "table_entries": wl.target_entries,
+            "between_steps": "L2 flushed (256 MiB write) and table restored to its seeded snapshot, untimed"}
+
+
+def run_reference(args, rank: int, world: int) -> None:
+    if rank != 0:
+        return
+    from paper_2609_38706_gb300 import workloads as W
+    import oracle as O
+    wl = W.FULL_CONFIGS[args.workload]()
+    d_ref, table = oracle_setup(wl)
+    n0 = len(table)
+    for _ in range(args.warmup):
+        cpu_oracle_pass(wl, d_ref, table, n0)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        cpu_oracle_pass(wl, d_ref, table, n0)
+    el = time.perf_counter() - t0
+    value = wl.tokens_keyed() * args.steps / el
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": 0,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
+            "data": "synthetic", "config": workload_config(wl, args),
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": O.max_threads(), "kind": "oracle",
+                             "sample": f"each step one full pass of the {wl.name} batch"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="pk", choices=["pk", "reference"])
+    ap.add_argument("--workload", default="multi_adapter")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+
+    import torch
+    import torch.distributed as dist
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_38706_gb300 import pk
+    from paper_2609_38706_gb300 import workloads as W
+    from paper_2609_38706_gb300.service import KeyTable
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    wl = W.FULL_CONFIGS[args.workload]()
+    C = wl.chunk_tokens
+    b = wl.batch
+    stream = torch.cuda.current_stream()
+
+    # ---- table: seeded from the prior batch by the GPU path itself ----
+    kt = KeyTable(C, wl.capacity_log2, device=dev)
+    d0 = kt.digests(wl.descriptors)
+    pko, pkeys = kt.derive(wl.prior.tokens, wl.prior.tok_off, wl.prior.desc_idx, d0)
+    pko_h = pko.cpu().numpy()
+    seeds = W.seed_list(pkeys.cpu().numpy()[: int(pko_h[-1])], pko_h, wl.prior_chunks)
+    kt.seed(seeds, wl.filler, wl.target_entries)
+    del pkeys, pko
+    snapshot = kt.save()
+
+    # ---- resident inputs and outputs ----
+    R, N_cap = b.R, b.n_tokens // C
+    tokens_h = torch.from_numpy(b.tokens).pin_memory()
+    tok_off_h = torch.from_numpy(b.tok_off).pin_memory()
+    desc_idx_h = torch.from_numpy(b.desc_idx.view(np.int32)).pin_memory()
+    tokens_d, tok_off_d, desc_idx_d = tokens_h.to(dev), tok_off_h.to(dev), desc_idx_h.to(dev)
+    descs = pk.Descriptors(wl.descriptors)
+    enc_h = torch.zeros(256 * 1024, dtype=torch.uint8).pin_memory()
+    enc_off_h = torch.zeros(descs.count + 1, dtype=torch.int64).pin_memory()
+    enc_used, _ = pk.pk_descriptors_encode(descs, enc_h.numpy(), enc_off_h.numpy())
+    n_enc = int(enc_used.size)
+    enc_d = torch.zeros(n_enc, dtype=torch.uint8, device=dev)
+    enc_off_d = torch.zeros(descs.count + 1, dtype=torch.int64, device=dev)
+    digests_d = torch.zeros((descs.count, 32), dtype=torch.uint8, device=dev)
+    key_off_d = torch.empty(R + 1, dtype=torch.int64, device=dev)
+    keys_d = torch.empty((N_cap, 32), dtype=torch.uint8, device=dev)
+    hit_d = torch.empty(R, dtype=torch.int32, device=dev)
+    slots_d = torch.empty(N_cap, dtype=torch.int32, device=dev)
+    new_slots_d = torch.arange(N_cap, dtype=torch.int32, device=dev) + (1 << 30)
+    result_d = torch.empty(N_cap, dtype=torch.int32, device=dev)
+    slot_out_d = torch.empty(N_cap, dtype=torch.int32, device=dev)
+    hit_h = torch.empty(R, dtype=torch.int32).pin_memory()
+    slots_h = torch.empty(N_cap, dtype=torch.int32).pin_memory()
+    result_h = torch.empty(N_cap, dtype=torch.int32).pin_memory()
+    slot_out_h = torch.empty(N_cap, dtype=torch.int32).pin_memory()
+    status = kt.status
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    ctx = kt.ctx
+
+    def core(ev=None):
+        pk.pk_descriptors_encode(descs, enc_h.numpy(), enc_off_h.numpy())      # a0, host
+        enc_d.copy_(enc_h[:n_enc], non_blocking=True)
+        enc_off_d.copy_(enc_off_h, non_blocking=True)
+        pk.pk_digest_descriptors(ctx, enc_d, enc_off_d, digests_d, status)     # a0, device
+        if ev: ev[1].record(stream)
+        pk.pk_derive_keys(ctx, tokens_d, tok_off_d, desc_idx_d, digests_d, key_off_d, keys_d, status)  # a1, a2
+        if ev: ev[2].record(stream)
+        pk.pk_lookup(ctx, keys_d, key_off_d, hit_d, slots_d, status)           # a3
+        if ev: ev[3].record(stream)
+        pk.pk_store(ctx, keys_d, new_slots_d, result_d, slot_out_d, status, key_off_d, hit_d)  # a4
+
+    def between_steps():
+        kt.load(snapshot)
+        flush.fill_(1)
+
+    spin_cycles = int(300e-6 * 2.0e9)
+    n_keys = wl.n_keys()
+
+    # ---- warm-up, then timed device-resident steps ----
+    for _ in range(args.warmup):
+        between_steps()
+        core()
+    torch.cuda.synchronize()
+    if kt.take_status() != 0:
+        raise RuntimeError("device status after warm-up")
+    hit_ref = hit_d.cpu().numpy().copy()
+
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.start()
+    step_ms, derive_ms, lookup_ms, store_ms, a0_ms = [], [], [], [], []
+    for _ in range(args.steps):
+        between_steps()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+        torch.cuda._sleep(spin_cycles)
+        ev[0].record(stream)
+        core(ev)
+        ev[4].record(stream)
+        torch.cuda.synchronize()
+        step_ms.append(ev[0].elapsed_time(ev[4]))
+        a0_ms.append(ev[0].elapsed_time(ev[1]))
+        derive_ms.append(ev[1].elapsed_time(ev[2]))
+        lookup_ms.append(ev[2].elapsed_time(ev[3]))
+        store_ms.append(ev[3].elapsed_time(ev[4]))
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    if kt.take_status() != 0:
+        raise RuntimeError("device status after timed steps")
+    if not np.array_equal(hit_d.cpu().numpy(), hit_ref):
+        raise RuntimeError("hit lengths changed between steps")
+
+    # ---- e2e: host buffers, copies inside the timed region ----
+    e2e_ms = []
+    for i in range(args.warmup + args.steps):
+        between_steps()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        tokens_d.copy_(tokens_h, non_blocking=True)
+        tok_off_d.copy_(tok_off_h, non_blocking=True)
+        desc_idx_d.copy_(desc_idx_h, non_blocking=True)
+        core()
+        hit_h.copy_(hit_d, non_blocking=True)
+        slots_h.copy_(slots_d, non_blocking=True)
+        result_h.copy_(result_d, non_blocking=True)
+        slot_out_h.copy_(slot_out_d, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if i >= args.warmup:
+            e2e_ms.append(e0.elapsed_time(e1))
+    h2d = tokens_h.numel() * 4 + tok_off_h.numel() * 8 + desc_idx_h.numel() * 4 + n_enc + enc_off_h.numel() * 8
+    d2h = (hit_h.numel() + slots_h.numel() + result_h.numel() + slot_out_h.numel()) * 4
+
+    total_ms = float(np.sum(step_ms))
+    e2e_total = float(np.sum(e2e_ms))
+    if world > 1:
+        t = torch.tensor([total_ms, e2e_total], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms, e2e_total = float(t[0]), float(t[1])
+    tokens_per_step = wl.tokens_keyed()
+    value = tokens_per_step * args.steps * world / (total_ms / 1e3)
+    e2e_value = tokens_per_step * args.steps * world / (e2e_total / 1e3)
+
+    peaks = load_peaks()
+    c_dig, c_chain = compressions(n_keys, C)
+    derive_s = float(np.mean(derive_ms)) / 1e3
+    alu_peak = SMS * LANES_PER_SM * peaks["sm_max_mhz"] * 1e6 / 1e12           # Tops/s
+    achieved = (c_dig + c_chain) * SHA_OPS_PER_COMPRESSION / derive_s / 1e12
+    lookup_s = float(np.mean(lookup_ms)) / 1e3
+    probe_bytes = n_keys * (16 + 32 + 4) + R * 4
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
+        "config": workload_config(wl, args),
+        "lookups_per_s": n_keys * args.steps * world / (total_ms / 1e3),
+        "requests_per_s": R * args.steps * world / (total_ms / 1e3),
+        "phase_ms": {"a0_descriptors": float(np.mean(a0_ms)), "derive_keys": float(np.mean(derive_ms)),
+                     "lookup": float(np.mean(lookup_ms)), "store": float(np.mean(store_ms))},
+        "roofline": {"bound": "alu", "kernel": "pk_derive_keys (chunk offsets + chunk digests + chain)",
+                     "achieved": achieved, "peak": alu_peak, "unit": "Tops/s", "frac": achieved / alu_peak,
+                     "traffic": None,
+                     "peak_basis": f"{SMS} SMs x {LANES_PER_SM} int32 lanes x {peaks['sm_max_mhz']:.0f} MHz "
+                                   f"(issue-rate ceiling); {SHA_OPS_PER_COMPRESSION} ops per compression, "
+                                   f"{c_dig + c_chain} compressions per launch"},
+        "probe_roofline": {"bound": "hbm", "kernel": "pk_lookup", "achieved": probe_bytes / lookup_s / 1e9,
+                           "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                           "frac": probe_bytes / lookup_s / 1e9 / peaks["hbm_gbs"],
+                           "bytes_basis": "per probe 16 B key + one 32 B entry sector + 4 B slot; 4 B per request",
+                           "peak_source": peaks["source"]},
+        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_total / args.steps},
+        "gpu_launches": 8 * args.steps,
+        "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = run_cpu_baseline(wl, args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    kt.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,215 @@
+/*
+ * pk.h -- C ABI of libpk: provenance-bound KV-cache keys on one GPU.
+ *
+ * The paper ("Preserving Provenance in Shared KV Caches for LLM Serving")
+ * requires a shared KV tier's key to be injective over every declared
+ * provenance dimension (Def. 2, Eqs. 1 and 2) and realises it as
+ *     Key(x, c) = f(x, H(enc(id_1(c(d_1)), ..., id_n(c(d_n)))))      (Eq. 3)
+ * This library computes that key for a batch of requests and keeps a
+ * GPU-resident table of key prefixes, with
+ *     H   = SHA-256,  d = H(enc(canonical descriptor))
+ *     f   = chained per-chunk digest:
+ *           c_i = SHA-256(int32 little-endian bytes of tokens[iC, (i+1)C))
+ *           k_i = SHA-256(k_{i-1} || d || c_i),   k_{-1} = 32 zero bytes
+ * over the floor(T/C) full chunks of each request (a partial trailing chunk
+ * gets no key; Sec. 4.4).  The table maps the first 16 bytes of k_i (the
+ * 128-bit digest width of Sec. 5.3) to a uint32 chunk slot.  Lookup returns
+ * each request's longest all-hit prefix; store inserts the misses (Sec. 2.1:
+ * on a local miss the connector queries the store; a hit skips that prefill,
+ * a miss computes and writes new state).  Lookup and store consume keys from
+ * one pk_derive_keys call, so both sites derive keys from the same
+ * descriptor value (Sec. 5.3, "Cross-site consistency").
+ *
+ * Conventions for every call
+ *   - Returns PK_OK (0) or a negative PK_ERR_* code.  A host-detected error
+ *     returns before anything is enqueued and leaves the table unchanged.
+ *   - "_dev" pointers are device memory owned by the caller; the library
+ *     allocates no device memory except a small fixed block in pk_init.
+ *   - All device work is enqueued asynchronously on the given stream
+ *     (NULL = legacy default stream).  Errors found on the device are written
+ *     to the caller's int32 status word *status_dev (first error wins; the
+ *     caller zeroes it and reads it after synchronising).  After a device
+ *     error the call's outputs are unspecified, but no access leaves the
+ *     caller's buffers and no wait is unbounded.
+ *   - A context is not thread-safe; calls on one context must be ordered.
+ */
+#ifndef PK_H_
+#define PK_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+#define PK_OK 0
+#define PK_ERR_ARG (-1)            /* null / misaligned pointer, bad size, bad offsets or index */
+#define PK_ERR_CAPACITY (-2)       /* capacity not a power of two in [2, 2^31], or table too small */
+#define PK_ERR_UNRESOLVED (-3)     /* precision or KV format empty or "auto" (Sec. 5.3) */
+#define PK_ERR_FIELD_TOO_LONG (-4) /* a descriptor field over PK_MAX_FIELD_BYTES */
+#define PK_ERR_TABLE_FULL (-5)     /* insertion would leave no empty slot */
+#define PK_ERR_PROBE_LIMIT (-6)    /* probe sequence longer than max_probe */
+#define PK_ERR_RESERVED_KEY (-7)   /* key prefix is all zero (the empty marker), p = 2^-128 */
+#define PK_ERR_CUDA (-8)           /* a CUDA runtime call or launch failed */
+
+/* Per-entry store results (int32). Negative values are the error codes above. */
+#define PK_STORE_SKIPPED 0         /* not in a miss range (range mode) */
+#define PK_STORE_INSERTED 1        /* new key; the entry's own slot was stored */
+#define PK_STORE_PRESENT 2         /* key already present (or an earlier duplicate in the batch won) */
+
+#define PK_NO_SLOT 0xFFFFFFFFu     /* lookup miss; not a storable slot value */
+#define PK_MAX_FIELD_BYTES 4096u
+#define PK_KEY_BYTES 32u           /* one full key k_i */
+#define PK_PREFIX_BYTES 16u        /* table key = first 16 bytes of k_i */
+#define PK_ENTRY_BYTES 32u         /* one table entry in device memory */
+
+typedef struct pk_ctx pk_ctx;
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st *pk_stream;
+
+/* A byte string; p may be NULL when len == 0. */
+typedef struct {
+    const uint8_t *p;
+    uint32_t len;
+} pk_bytes;
+
+/* One provenance descriptor: registry v1 in encoding order (Sec. 5.1 dimensions
+ * plus the model identity, Sec. 5.3), then optional appended dimensions
+ * (Prop. 1: appending a well-formed dimension preserves the contract).
+ * Empty adapter_id / salt mean "none".  weight_precision and kv_format must be
+ * resolved values (ASCII case-insensitive; bfloat16->bf16, float16|half->fp16,
+ * float32|float->fp32, float8_e4m3fn->fp8_e4m3, float8_e5m2->fp8_e5m2; any
+ * other spelling is kept as written).  Other fields are opaque bytes. */
+typedef struct {
+    pk_bytes model_id;
+    pk_bytes weight_precision;
+    pk_bytes weight_version;
+    pk_bytes adapter_id;
+    pk_bytes kv_format;
+    pk_bytes salt;
+    const pk_bytes *extra; /* n_extra appended dimension identities, or NULL */
+    uint32_t n_extra;
+} pk_descriptor;
+
+typedef struct {
+    uint32_t chunk_tokens;  /* C >= 1 */
+    uint32_t capacity_log2; /* table capacity = 2^capacity_log2, 1..31 */
+    uint32_t max_probe;     /* probe sequence bound per key; 0 = capacity */
+    void *table_dev;        /* caller-owned, 16-byte aligned */
+    size_t table_bytes;     /* >= pk_table_bytes(capacity_log2) */
+} pk_config;
+
+/* Bytes of device memory a table of 2^capacity_log2 entries needs (0 if out of range). */
+size_t pk_table_bytes(uint32_t capacity_log2);
+
+/* Create a context bound to the caller's table and clear the table (all
+ * entries empty) on `stream`.  Allocates one small device block (entry
+ * counter).  *out is NULL on error.  Errors: PK_ERR_ARG, PK_ERR_CAPACITY,
+ * PK_ERR_CUDA. */
+int pk_init(pk_ctx **out, const pk_config *cfg, pk_stream stream);
+
+/* Release the context (not the caller's table).  Synchronises nothing;
+ * the caller must not destroy a context with work still in flight. */
+int pk_destroy(pk_ctx *ctx);
+
+/* Host.  Canonicalise one descriptor and write enc = LE32(field count) ||
+ * (LE32(len) || bytes) per field (Sec. 5.2: injective, length-prefixed) into
+ * out[0, cap).  *len receives the encoded size (also when cap is too small,
+ * in which case PK_ERR_ARG is returned).  Errors: PK_ERR_ARG,
+ * PK_ERR_UNRESOLVED, PK_ERR_FIELD_TOO_LONG. */
+int pk_descriptor_encode(const pk_descriptor *desc, uint8_t *out, size_t cap, size_t *len);
+
+/* Host.  Encode D descriptors back to back; enc_off (D+1 entries) receives the
+ * byte offsets.  Same errors as pk_descriptor_encode (first failing one). */
+int pk_descriptors_encode(const pk_descriptor *descs, uint32_t D, uint8_t *out, size_t cap,
+                          int64_t *enc_off);
+
+/* Host.  d = SHA-256(enc(canonical descriptor)) (Eq. 3, H over enc). */
+int pk_descriptor_digest(const pk_descriptor *desc, uint8_t out[32]);
+
+/* Device.  digests_dev[j] = SHA-256(enc_dev[enc_off_dev[j], enc_off_dev[j+1]))
+ * for j < D: the descriptor digests d of a batch (Eq. 3, H over enc), from
+ * encodings produced by pk_descriptors_encode and copied to the device.
+ * enc_dev holds enc_bytes bytes; enc_off_dev holds D+1 offsets; digests_dev:
+ * D*32 bytes.  Device errors (offsets decreasing or beyond enc_bytes):
+ * PK_ERR_ARG in *status_dev, that digest left unwritten. */
+int pk_digest_descriptors(pk_ctx *ctx, const uint8_t *enc_dev, uint64_t enc_bytes,
+                          const int64_t *enc_off_dev, uint32_t D, uint8_t *digests_dev,
+                          int32_t *status_dev, pk_stream stream);
+
+/* Device.  Key derivation for R requests (steps c_i and k_i above).
+ *   tokens_dev   int32[n_tokens]
+ *   tok_off_dev  int64[R+1], non-decreasing, tok_off[R] <= n_tokens;
+ *                request r = tokens[tok_off[r], tok_off[r+1])
+ *   desc_idx_dev uint32[R] < D;  digests_dev uint8[D*32] (16-byte aligned)
+ *   key_off_dev  OUT int64[R+1]: key_off[0] = 0,
+ *                key_off[r+1] = key_off[r] + floor((tok_off[r+1]-tok_off[r]) / C)
+ *   keys_dev     OUT uint8[key_capacity*32] (16-byte aligned): key j of
+ *                request r at index key_off[r] + j.  key_capacity must be at
+ *                least floor(n_tokens / C), which always suffices.
+ * Any request layout is accepted (starts need not be aligned).  Device errors
+ * (offsets not monotone or out of range, desc_idx >= D): PK_ERR_ARG in
+ * *status_dev and key_off all zero. */
+int pk_derive_keys(pk_ctx *ctx, const int32_t *tokens_dev, uint64_t n_tokens,
+                   const int64_t *tok_off_dev, uint32_t R, const uint32_t *desc_idx_dev,
+                   const uint8_t *digests_dev, uint32_t D, int64_t *key_off_dev,
+                   uint8_t *keys_dev, uint64_t key_capacity, int32_t *status_dev,
+                   pk_stream stream);
+
+/* Device.  Probe the table for every key of a pk_derive_keys result.
+ *   slots_dev       OUT uint32[key_capacity]: slot of key i, or PK_NO_SLOT
+ *   hit_chunks_dev  OUT int32[R]: h_r = the largest j such that keys 0..j-1 of
+ *                   request r are all present (the first miss ends the prefix);
+ *                   the keys to store are those of [h_r, n_r)
+ * The table is read as of the start of the call.  Device errors:
+ * PK_ERR_PROBE_LIMIT (that key reads as a miss). */
+int pk_lookup(pk_ctx *ctx, const uint8_t *keys_dev, const int64_t *key_off_dev, uint32_t R,
+              uint64_t key_capacity, int32_t *hit_chunks_dev, uint32_t *slots_dev,
+              int32_t *status_dev, pk_stream stream);
+
+/* Device.  Insert-if-absent of (prefix of keys_dev[e], slots_dev[e]), with
+ * the outcome of processing the entries one by one in index order: an absent
+ * key is inserted with its own slot (PK_STORE_INSERTED); a key already in the
+ * table, or inserted by a lower index of the same call, keeps the existing
+ * slot (PK_STORE_PRESENT).  slot_out_dev[e] receives the slot now bound to the
+ * key (PK_NO_SLOT for skipped or failed entries).
+ *   list mode  (key_off_dev == NULL, hit_chunks_dev == NULL): entries 0..n-1
+ *   range mode (both given, R requests): only the miss ranges
+ *              [key_off[r] + hit_chunks[r], key_off[r+1]) of a pk_lookup
+ *              result; n = key_capacity; other entries get PK_STORE_SKIPPED.
+ * keys_dev: n*32 bytes (only the first 16 of each used), 16-byte aligned;
+ * slots_dev: uint32[n], values != PK_NO_SLOT; result_dev: int32[n];
+ * slot_out_dev: uint32[n] (required: also holds intermediate positions).
+ * Per-entry errors: PK_ERR_RESERVED_KEY, PK_ERR_ARG (slot == PK_NO_SLOT),
+ * PK_ERR_TABLE_FULL, PK_ERR_PROBE_LIMIT; the first one also goes to
+ * *status_dev.  Near capacity, which of a call's new keys are refused is
+ * unspecified. */
+int pk_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_dev, uint64_t n,
+             const int64_t *key_off_dev, const int32_t *hit_chunks_dev, uint32_t R,
+             int32_t *result_dev, uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream);
+
+/* Checkpoint (the shared store outlives workers, Sec. 2.1).  Asynchronous on
+ * `stream`: copies the table and its entry count to dst (device or host
+ * memory, dst_bytes >= pk_table_bytes(capacity_log2) + 64). */
+int pk_table_save(pk_ctx *ctx, void *dst, size_t dst_bytes, pk_stream stream);
+
+/* Resume: replace this context's table with one saved by pk_table_save from a
+ * context of the same capacity (src: device or host memory, src_bytes >=
+ * pk_table_bytes + 64).  Keys and slots are restored exactly; the entries
+ * count as inserted before any later store call.  Asynchronous on `stream`. */
+int pk_table_load(pk_ctx *ctx, const void *src, size_t src_bytes, pk_stream stream);
+
+/* Host, synchronous.  Number of entries in the table (device counter read
+ * after synchronising `stream`). */
+int pk_entries(pk_ctx *ctx, uint64_t *count, pk_stream stream);
+
+/* Static description of a status code. */
+const char *pk_strerror(int code);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PK_H_ */

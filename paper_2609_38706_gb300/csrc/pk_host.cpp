@@ -1,0 +1,265 @@
+// pk_host.cpp -- host half of libpk: argument checks, descriptor
+// canonicalisation and enc (Sec. 5.2-5.3), the host descriptor digest, and
+// the C-ABI entry points that enqueue the kernels of pk_derive.cu / pk_table.cu.
+#include <cuda_runtime_api.h>
+
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <string>
+
+#include "pk_internal.h"
+#include "pk_sha256.cuh"
+
+namespace {
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Sec. 5.3, worker-level digest: bind the value the worker resolved, never a
+// launch string such as "auto".  Resolved dtype names are compared ASCII
+// case-insensitively and exact synonyms are folded to one spelling; distinct
+// formats are never merged (a bare "fp8" stays "fp8").
+int canonical_dtype(const pk_bytes &in, std::string *out) {
+    if (in.len > PK_MAX_FIELD_BYTES) return PK_ERR_FIELD_TOO_LONG;
+    if (in.len && !in.p) return PK_ERR_ARG;
+    std::string s(reinterpret_cast<const char *>(in.p), in.len);
+    for (char &c : s)
+        if (c >= 'A' && c <= 'Z') c = (char)(c + 32);
+    static const char *const kSyn[][2] = {
+        {"bfloat16", "bf16"},          {"float16", "fp16"},         {"half", "fp16"},
+        {"float32", "fp32"},           {"float", "fp32"},           {"float8_e4m3fn", "fp8_e4m3"},
+        {"float8_e5m2", "fp8_e5m2"},
+    };
+    for (const auto &kv : kSyn)
+        if (s == kv[0]) {
+            s = kv[1];
+            break;
+        }
+    if (s.empty() || s == "auto") return PK_ERR_UNRESOLVED;
+    *out = s;
+    return PK_OK;
+}
+
+int opaque(const pk_bytes &in, std::string *out) {
+    if (in.len > PK_MAX_FIELD_BYTES) return PK_ERR_FIELD_TOO_LONG;
+    if (in.len && !in.p) return PK_ERR_ARG;
+    out->assign(reinterpret_cast<const char *>(in.p), in.len);
+    return PK_OK;
+}
+
+void put_le32(std::string *dst, uint32_t v) {
+    const char b[4] = {(char)(v & 0xff), (char)((v >> 8) & 0xff), (char)((v >> 16) & 0xff), (char)(v >> 24)};
+    dst->append(b, 4);
+}
+
+// enc: LE32(number of fields) || for each field LE32(length) || bytes
+// (Sec. 5.2, Eq. 3: injective, length-prefixed; appended fields per Prop. 1).
+int encode(const pk_descriptor *d, std::string *enc) {
+    if (!d) return PK_ERR_ARG;
+    if (d->n_extra && !d->extra) return PK_ERR_ARG;
+    std::string f[6];
+    int rc;
+    if ((rc = opaque(d->model_id, &f[0])) != PK_OK) return rc;
+    if ((rc = canonical_dtype(d->weight_precision, &f[1])) != PK_OK) return rc;
+    if ((rc = opaque(d->weight_version, &f[2])) != PK_OK) return rc;
+    if ((rc = opaque(d->adapter_id, &f[3])) != PK_OK) return rc;
+    if ((rc = canonical_dtype(d->kv_format, &f[4])) != PK_OK) return rc;
+    if ((rc = opaque(d->salt, &f[5])) != PK_OK) return rc;
+    enc->clear();
+    put_le32(enc, 6u + d->n_extra);
+    for (const auto &s : f) {
+        put_le32(enc, (uint32_t)s.size());
+        enc->append(s);
+    }
+    for (uint32_t j = 0; j < d->n_extra; ++j) {
+        std::string x;
+        if ((rc = opaque(d->extra[j], &x)) != PK_OK) return rc;
+        put_le32(enc, (uint32_t)x.size());
+        enc->append(x);
+    }
+    return PK_OK;
+}
+
+int cuda_rc(cudaError_t e) { return e == cudaSuccess ? PK_OK : PK_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+size_t pk_table_bytes(uint32_t capacity_log2) {
+    if (capacity_log2 < 1 || capacity_log2 > 31) return 0;
+    return (size_t)PK_ENTRY_BYTES << capacity_log2;
+}
+
+int pk_init(pk_ctx **out, const pk_config *cfg, pk_stream stream) {
+    if (!out) return PK_ERR_ARG;
+    *out = nullptr;
+    if (!cfg || cfg->chunk_tokens == 0 || !cfg->table_dev || !aligned16(cfg->table_dev)) return PK_ERR_ARG;
+    const size_t need = pk_table_bytes(cfg->capacity_log2);
+    if (need == 0 || cfg->table_bytes < need) return PK_ERR_CAPACITY;
+    pk_ctx *c = new (std::nothrow) pk_ctx();
+    if (!c) return PK_ERR_ARG;
+    c->chunk_tokens = cfg->chunk_tokens;
+    c->capacity_log2 = cfg->capacity_log2;
+    c->capacity = 1ull << cfg->capacity_log2;
+    c->max_probe = (cfg->max_probe == 0 || cfg->max_probe > c->capacity) ? (uint32_t)c->capacity : cfg->max_probe;
+    c->table = static_cast<pk_entry *>(cfg->table_dev);
+    c->epoch = 0;
+    if (cudaMalloc(reinterpret_cast<void **>(&c->counter_dev), 256) != cudaSuccess) {
+        delete c;
+        return PK_ERR_CUDA;
+    }
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemsetAsync(c->table, 0, need, s) != cudaSuccess ||
+        cudaMemsetAsync(c->counter_dev, 0, 256, s) != cudaSuccess) {
+        cudaFree(c->counter_dev);
+        delete c;
+        return PK_ERR_CUDA;
+    }
+    *out = c;
+    return PK_OK;
+}
+
+int pk_destroy(pk_ctx *ctx) {
+    if (!ctx) return PK_ERR_ARG;
+    const cudaError_t e = cudaFree(ctx->counter_dev);
+    delete ctx;
+    return cuda_rc(e);
+}
+
+int pk_descriptor_encode(const pk_descriptor *desc, uint8_t *out, size_t cap, size_t *len) {
+    std::string enc;
+    const int rc = encode(desc, &enc);
+    if (rc != PK_OK) return rc;
+    if (len) *len = enc.size();
+    if (enc.size() > cap || (!out && !enc.empty())) return PK_ERR_ARG;
+    std::memcpy(out, enc.data(), enc.size());
+    return PK_OK;
+}
+
+int pk_descriptors_encode(const pk_descriptor *descs, uint32_t D, uint8_t *out, size_t cap, int64_t *enc_off) {
+    if (!enc_off || (D && !descs)) return PK_ERR_ARG;
+    enc_off[0] = 0;
+    size_t pos = 0;
+    std::string enc;
+    for (uint32_t j = 0; j < D; ++j) {
+        const int rc = encode(descs + j, &enc);
+        if (rc != PK_OK) return rc;
+        if (pos + enc.size() > cap || !out) return PK_ERR_ARG;
+        std::memcpy(out + pos, enc.data(), enc.size());
+        pos += enc.size();
+        enc_off[j + 1] = (int64_t)pos;
+    }
+    return PK_OK;
+}
+
+int pk_descriptor_digest(const pk_descriptor *desc, uint8_t out[32]) {
+    if (!out) return PK_ERR_ARG;
+    std::string enc;
+    const int rc = encode(desc, &enc);
+    if (rc != PK_OK) return rc;
+    pk::sha256_bytes(reinterpret_cast<const uint8_t *>(enc.data()), enc.size(), out);
+    return PK_OK;
+}
+
+int pk_digest_descriptors(pk_ctx *ctx, const uint8_t *enc_dev, uint64_t enc_bytes, const int64_t *enc_off_dev,
+                          uint32_t D, uint8_t *digests_dev, int32_t *status_dev, pk_stream stream) {
+    if (!ctx) return PK_ERR_ARG;
+    if (D == 0) return PK_OK;
+    if (!enc_off_dev || !digests_dev || (enc_bytes && !enc_dev)) return PK_ERR_ARG;
+    return cuda_rc(pk_launch_digest_descriptors(enc_dev, enc_bytes, enc_off_dev, D, digests_dev, status_dev,
+                                                reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int pk_derive_keys(pk_ctx *ctx, const int32_t *tokens_dev, uint64_t n_tokens, const int64_t *tok_off_dev,
+                   uint32_t R, const uint32_t *desc_idx_dev, const uint8_t *digests_dev, uint32_t D,
+                   int64_t *key_off_dev, uint8_t *keys_dev, uint64_t key_capacity, int32_t *status_dev,
+                   pk_stream stream) {
+    if (!ctx || !tok_off_dev || !key_off_dev) return PK_ERR_ARG;
+    if (n_tokens && !tokens_dev) return PK_ERR_ARG;
+    if (R && (!desc_idx_dev || !digests_dev || D == 0 || !aligned16(digests_dev))) return PK_ERR_ARG;
+    if (key_capacity < n_tokens / ctx->chunk_tokens) return PK_ERR_ARG;
+    if (key_capacity && (!keys_dev || !aligned16(keys_dev))) return PK_ERR_ARG;
+    if (key_capacity > (uint64_t)0x7fffffff * 64) return PK_ERR_ARG;
+    return cuda_rc(pk_launch_derive(ctx, tokens_dev, n_tokens, tok_off_dev, R, desc_idx_dev, digests_dev, D,
+                                    key_off_dev, keys_dev, key_capacity, status_dev,
+                                    reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int pk_lookup(pk_ctx *ctx, const uint8_t *keys_dev, const int64_t *key_off_dev, uint32_t R,
+              uint64_t key_capacity, int32_t *hit_chunks_dev, uint32_t *slots_dev, int32_t *status_dev,
+              pk_stream stream) {
+    if (!ctx || !key_off_dev) return PK_ERR_ARG;
+    if (R && !hit_chunks_dev) return PK_ERR_ARG;
+    if (key_capacity && (!keys_dev || !aligned16(keys_dev) || !slots_dev)) return PK_ERR_ARG;
+    if (key_capacity > (uint64_t)0x7fffffff * 256) return PK_ERR_ARG;
+    return cuda_rc(pk_launch_lookup(ctx, keys_dev, key_off_dev, R, key_capacity, hit_chunks_dev, slots_dev,
+                                    status_dev, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int pk_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_dev, uint64_t n,
+             const int64_t *key_off_dev, const int32_t *hit_chunks_dev, uint32_t R, int32_t *result_dev,
+             uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream) {
+    if (!ctx) return PK_ERR_ARG;
+    if ((key_off_dev == nullptr) != (hit_chunks_dev == nullptr)) return PK_ERR_ARG;
+    if (n == 0) return PK_OK;
+    if (!keys_dev || !aligned16(keys_dev) || !slots_dev || !result_dev || !slot_out_dev) return PK_ERR_ARG;
+    if (n > (uint64_t)0x7fffffff * 256 || n >= 0xffffffffull) return PK_ERR_ARG;
+    const unsigned long long epoch = ++ctx->epoch;
+    return cuda_rc(pk_launch_store(ctx, epoch, keys_dev, slots_dev, n, key_off_dev, hit_chunks_dev,
+                                   key_off_dev ? R : 0, result_dev, slot_out_dev, status_dev,
+                                   reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int pk_table_save(pk_ctx *ctx, void *dst, size_t dst_bytes, pk_stream stream) {
+    if (!ctx || !dst) return PK_ERR_ARG;
+    const size_t tb = pk_table_bytes(ctx->capacity_log2);
+    if (dst_bytes < tb + 64) return PK_ERR_ARG;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(dst, ctx->table, tb, cudaMemcpyDefault, s) != cudaSuccess ||
+        cudaMemcpyAsync(static_cast<uint8_t *>(dst) + tb, ctx->counter_dev, sizeof(unsigned long long),
+                        cudaMemcpyDefault, s) != cudaSuccess)
+        return PK_ERR_CUDA;
+    return PK_OK;
+}
+
+int pk_table_load(pk_ctx *ctx, const void *src, size_t src_bytes, pk_stream stream) {
+    if (!ctx || !src) return PK_ERR_ARG;
+    const size_t tb = pk_table_bytes(ctx->capacity_log2);
+    if (src_bytes < tb + 64) return PK_ERR_ARG;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(ctx->table, src, tb, cudaMemcpyDefault, s) != cudaSuccess ||
+        cudaMemcpyAsync(ctx->counter_dev, static_cast<const uint8_t *>(src) + tb, sizeof(unsigned long long),
+                        cudaMemcpyDefault, s) != cudaSuccess)
+        return PK_ERR_CUDA;
+    if (ctx->epoch < 1) ctx->epoch = 1;
+    return cuda_rc(pk_launch_mark_loaded(ctx, s));
+}
+
+int pk_entries(pk_ctx *ctx, uint64_t *count, pk_stream stream) {
+    if (!ctx || !count) return PK_ERR_ARG;
+    unsigned long long v = 0;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(&v, ctx->counter_dev, sizeof v, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return PK_ERR_CUDA;
+    *count = v;
+    return PK_OK;
+}
+
+const char *pk_strerror(int code) {
+    switch (code) {
+        case PK_OK: return "ok";
+        case PK_ERR_ARG: return "invalid argument";
+        case PK_ERR_CAPACITY: return "capacity not a power of two in [2, 2^31] or table buffer too small";
+        case PK_ERR_UNRESOLVED: return "weight precision or KV format is empty or unresolved (auto)";
+        case PK_ERR_FIELD_TOO_LONG: return "descriptor field longer than PK_MAX_FIELD_BYTES";
+        case PK_ERR_TABLE_FULL: return "table full";
+        case PK_ERR_PROBE_LIMIT: return "probe limit reached";
+        case PK_ERR_RESERVED_KEY: return "key prefix is the reserved all-zero value";
+        case PK_ERR_CUDA: return "CUDA runtime error";
+        default: return "unknown status";
+    }
+}
+
+}  // extern "C"

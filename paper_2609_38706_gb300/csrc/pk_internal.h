@@ -1,0 +1,49 @@
+// pk_internal.h -- context, table entry layout and kernel launchers of libpk.
+#pragma once
+#include <cuda_runtime_api.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/pk.h"
+
+// One table entry, 32 bytes (one DRAM sector):
+//   k[0..3]  the 16-byte key prefix, stored byte for byte (all zero = empty)
+//   slot     the chunk slot bound to the key
+//   owner    during a store call: ~(lowest entry index that claimed the key)
+//   epoch    number of the store call that inserted the key (0 while empty)
+struct alignas(32) pk_entry {
+    uint32_t k[4];
+    uint32_t slot;
+    uint32_t owner;
+    unsigned long long epoch;
+};
+static_assert(sizeof(pk_entry) == PK_ENTRY_BYTES, "entry layout");
+
+struct pk_ctx {
+    uint32_t chunk_tokens;
+    uint32_t capacity_log2;
+    uint32_t max_probe;
+    uint64_t capacity;
+    pk_entry *table;
+    unsigned long long *counter_dev;  // number of entries in the table
+    unsigned long long epoch;         // last store call number
+};
+
+// internal per-entry state between the two store kernels
+#define PK_STORE_PENDING 0x40000000
+
+// Launchers (pk_derive.cu, pk_table.cu).  Each returns the launch error.
+cudaError_t pk_launch_digest_descriptors(const uint8_t *enc, uint64_t enc_bytes, const int64_t *enc_off,
+                                         uint32_t D, uint8_t *digests, int32_t *status, cudaStream_t s);
+cudaError_t pk_launch_derive(const pk_ctx *ctx, const int32_t *tokens, uint64_t n_tokens,
+                             const int64_t *tok_off, uint32_t R, const uint32_t *desc_idx,
+                             const uint8_t *digests, uint32_t D, int64_t *key_off, uint8_t *keys,
+                             uint64_t key_capacity, int32_t *status, cudaStream_t s);
+cudaError_t pk_launch_lookup(const pk_ctx *ctx, const uint8_t *keys, const int64_t *key_off, uint32_t R,
+                             uint64_t key_capacity, int32_t *hit_chunks, uint32_t *slots, int32_t *status,
+                             cudaStream_t s);
+cudaError_t pk_launch_mark_loaded(const pk_ctx *ctx, cudaStream_t s);
+cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const uint8_t *keys,
+                            const uint32_t *slots, uint64_t n, const int64_t *key_off,
+                            const int32_t *hit_chunks, uint32_t R, int32_t *result, uint32_t *slot_out,
+                            int32_t *status, cudaStream_t s);

@@ -1,0 +1,127 @@
+"""C-ABI checks that need no GPU: the library loads, exports every entry point
+include/pk.h declares, and its host-side steps (descriptor canonicalisation,
+enc and the descriptor digest d of Eq. 3) match the oracle exactly; host
+argument errors are reported before any CUDA call."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2609_38706_gb300 import _build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def pk():
+    _build.build()
+    from paper_2609_38706_gb300 import pk as pk_mod
+    pk_mod.lib()
+    return pk_mod
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "pk.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(pk_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("pk_init", "pk_derive_keys", "pk_lookup", "pk_store", "pk_destroy", "pk_descriptor_digest"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(pk):
+    L = ctypes.CDLL(_build.LIB)
+    missing = [n for n in declared_functions() if not hasattr(L, n)]
+    assert not missing, missing
+
+
+def test_status_vocabulary_matches_header(pk):
+    src = open(os.path.join(ROOT, "include", "pk.h")).read()
+    for name in ("PK_ERR_ARG", "PK_ERR_CAPACITY", "PK_ERR_UNRESOLVED", "PK_ERR_FIELD_TOO_LONG", "PK_ERR_TABLE_FULL",
+                 "PK_ERR_PROBE_LIMIT", "PK_ERR_RESERVED_KEY", "PK_STORE_INSERTED", "PK_STORE_PRESENT"):
+        m = re.search(r"#define %s \(?(-?\d+)\)?" % name, src)
+        assert m and int(m.group(1)) == getattr(pk, name) == getattr(O, name.replace("PK_STORE_", "STORE_"), getattr(pk, name))
+
+
+def _rand_desc(rng):
+    pick = lambda opts: opts[int(rng.integers(0, len(opts)))]
+    d = {"model_id": pick(["synthetic/model-7b", "Org/Model", "", "m" * 300]),
+         "weight_precision": pick(["bf16", "BF16", "bfloat16", "fp8", "fp8_e4m3", "float8_e4m3fn", "Half", "int4-awq"]),
+         "weight_version": bytes(rng.integers(0, 256, int(rng.integers(0, 50)), dtype=np.uint8)),
+         "adapter_id": pick(["", "adapter-00", "Adapter-00", "sha256:" + "ab" * 32]),
+         "kv_format": pick(["bf16", "fp16", "float16", "fp8_e5m2", "FP8_E4M3", "float32"]),
+         "salt": pick(["", "tenant-a", "été"])}
+    if rng.random() < 0.3:
+        d["extra"] = [bytes(rng.integers(0, 256, int(rng.integers(0, 9)), dtype=np.uint8))
+                      for _ in range(int(rng.integers(1, 4)))]
+    return d
+
+
+def test_descriptor_digest_matches_oracle(pk):
+    rng = np.random.default_rng(5)
+    for _ in range(500):
+        d = _rand_desc(rng)
+        assert pk.pk_descriptor_encode(d) == O.enc(O.canonicalize(d))
+        assert pk.pk_descriptor_digest(d) == O.descriptor_digest(d)
+
+
+def test_batch_encode_offsets(pk):
+    rng = np.random.default_rng(6)
+    descs = [_rand_desc(rng) for _ in range(64)]
+    enc, off = pk.pk_descriptors_encode(descs)
+    for j, d in enumerate(descs):
+        assert bytes(enc[off[j]:off[j + 1]]) == O.enc(O.canonicalize(d))
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("weight_precision", "auto", -3), ("kv_format", "AUTO", -3), ("kv_format", "", -3),
+    ("weight_precision", "", -3), ("salt", "x" * 4097, -4), ("model_id", "y" * 4097, -4),
+])
+def test_descriptor_errors_match_oracle(pk, field, value, code):
+    d = {"model_id": "m", "weight_precision": "bf16", "weight_version": "v", "adapter_id": "", "kv_format": "bf16",
+         "salt": ""}
+    d[field] = value
+    with pytest.raises(pk.PKError) as e:
+        pk.pk_descriptor_digest(d)
+    assert e.value.code == code
+    with pytest.raises(O.OracleError) as e2:
+        O.descriptor_digest(d)
+    assert e2.value.code == code
+
+
+def test_descriptor_field_limit_exact(pk):
+    d = {"model_id": "m", "weight_precision": "bf16", "kv_format": "bf16", "salt": "s" * 4096}
+    assert pk.pk_descriptor_digest(d) == O.descriptor_digest(d)
+
+
+def test_table_bytes(pk):
+    assert pk.pk_table_bytes(0) == 0 and pk.pk_table_bytes(32) == 0
+    assert pk.pk_table_bytes(1) == 64 and pk.pk_table_bytes(20) == 32 << 20
+
+
+def test_init_host_errors_before_any_cuda_call(pk):
+    L = pk.lib()
+    out = ctypes.c_void_p()
+    # bad capacity and too-small table: rejected on the host (pointer never dereferenced)
+    for log2, nbytes in ((0, 1 << 20), (32, 1 << 20), (10, 32 * 1024 - 1)):
+        cfg = pk.pk_config(256, log2, 0, 4096, nbytes)
+        assert L.pk_init(ctypes.byref(out), ctypes.byref(cfg), None) == pk.PK_ERR_CAPACITY
+        assert out.value is None
+    for cfg in (pk.pk_config(0, 10, 0, 4096, 1 << 20), pk.pk_config(256, 10, 0, 0, 1 << 20),
+                pk.pk_config(256, 10, 0, 4100, 1 << 20)):
+        assert L.pk_init(ctypes.byref(out), ctypes.byref(cfg), None) == pk.PK_ERR_ARG
+    assert L.pk_init(None, ctypes.byref(pk.pk_config(256, 10, 0, 4096, 1 << 20)), None) == pk.PK_ERR_ARG
+
+
+def test_null_context_rejected(pk):
+    L = pk.lib()
+    assert L.pk_lookup(None, None, None, 0, 0, None, None, None, None) == pk.PK_ERR_ARG
+    assert L.pk_store(None, None, None, 0, None, None, 0, None, None, None, None) == pk.PK_ERR_ARG
+    assert L.pk_derive_keys(None, None, 0, None, 0, None, None, 0, None, None, 0, None, None) == pk.PK_ERR_ARG
+    assert L.pk_destroy(None) == pk.PK_ERR_ARG
