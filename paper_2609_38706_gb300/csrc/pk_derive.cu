@@ -13,14 +13,13 @@
 // and overwritten in place by the chain, so derivation needs no scratch memory.
 #include <cuda_runtime.h>
 
+#include "pk_device.cuh"
 #include "pk_internal.h"
 #include "pk_sha256.cuh"
 
 namespace {
 
-__device__ __forceinline__ void set_status(int32_t *status, int32_t code) {
-    if (status) atomicCAS(status, 0, code);
-}
+using pk::set_status;
 
 // ---------------------------------------------------------------------------
 // Descriptor digests: one thread per descriptor.
@@ -101,17 +100,6 @@ k_chunk_offsets(const int64_t *__restrict__ tok_off, uint32_t R, uint64_t n_toke
     }
 }
 
-// index of the request whose key range [key_off[r], key_off[r+1]) holds g
-__device__ __forceinline__ uint32_t find_request(const int64_t *__restrict__ key_off, uint32_t R,
-                                                 int64_t g) {
-    uint32_t lo = 0, hi = R;  // key_off[lo] <= g < key_off[hi]
-    while (hi - lo > 1) {
-        const uint32_t mid = (lo + hi) >> 1;
-        if (__ldg(key_off + mid) <= g) lo = mid; else hi = mid;
-    }
-    return lo;
-}
-
 __device__ __forceinline__ void store_digest(uint8_t *dst, const uint32_t st[8]) {
     uint4 *q = reinterpret_cast<uint4 *>(dst);
     q[0] = make_uint4(pk::bswap32(st[0]), pk::bswap32(st[1]), pk::bswap32(st[2]), pk::bswap32(st[3]));
@@ -138,18 +126,23 @@ __device__ __forceinline__ void load_block(const int32_t *__restrict__ src, bool
 }
 
 // ---------------------------------------------------------------------------
-// Chunk digests: one thread per chunk.  CT > 0 fixes the chunk size at
-// compile time (the padding block is then a constant message whose schedule
-// the compiler folds); CT == 0 takes it at run time.
+// Chunk digests: one thread per chunk, 32 consecutive chunks per warp.  CT > 0
+// fixes the chunk size at compile time (the padding block is then a constant
+// message whose schedule the compiler folds); CT == 0 takes it at run time.
+// The next 64-byte block is loaded while the current one is compressed.
 // ---------------------------------------------------------------------------
 template <int CT>
 __global__ void __launch_bounds__(128)
 k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_off,
                const int64_t *__restrict__ key_off, uint32_t R, uint32_t C_rt,
                uint8_t *__restrict__ keys) {
+    if (R == 0) return;
     const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (R == 0 || g >= __ldg(key_off + R)) return;
-    const uint32_t r = find_request(key_off, R, g);
+    const int64_t g0 = g - (threadIdx.x & 31);
+    const int64_t total = __ldg(key_off + R);
+    if (g0 >= total) return;  // whole warp past the end
+    const uint32_t r = pk::lane_request(key_off, R, g0, total, g);
+    if (g >= total) return;
     const int64_t i = g - __ldg(key_off + r);
     const uint32_t C = CT > 0 ? (uint32_t)CT : C_rt;
     const int32_t *src = tokens + __ldg(tok_off + r) + i * (int64_t)C;
@@ -158,22 +151,25 @@ k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ t
     uint32_t st[8];
     pk::init_state(st);
     const uint32_t nfull = C / 16;
+    uint32_t w[16];
+    if (nfull > 0) load_block(src, aligned, w);
 #pragma unroll 1
     for (uint32_t b = 0; b < nfull; ++b) {
-        uint32_t w[16];
-        load_block(src + 16 * b, aligned, w);
+        uint32_t nx[16];
+        if (b + 1 < nfull) load_block(src + 16 * (b + 1), aligned, nx);
         pk::compress16(st, w);
+#pragma unroll
+        for (int t = 0; t < 16; ++t) w[t] = nx[t];
     }
     const uint64_t bits = (uint64_t)C * 32u;
-    const uint32_t rem = C % 16;
+    const int rem = (int)(C % 16);
     if (rem == 0) {
         pk::compress(st, 0x80000000u, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0,
                      (uint32_t)(bits >> 32), (uint32_t)bits);
     } else {
-        uint32_t w[16];
         const int32_t *tail = src + 16 * nfull;
 #pragma unroll
-        for (uint32_t t = 0; t < 16; ++t)
+        for (int t = 0; t < 16; ++t)
             w[t] = t < rem ? pk::bswap32((uint32_t)__ldg(tail + t)) : (t == rem ? 0x80000000u : 0u);
         if (rem <= 13) {
             w[14] = (uint32_t)(bits >> 32);

@@ -14,6 +14,8 @@
 namespace {
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+// typed arrays must be naturally aligned (NULL passes; presence is checked separately)
+bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
 // Sec. 5.3, worker-level digest: bind the value the worker resolved, never a
 // launch string such as "auto".  Resolved dtype names are compared ASCII
@@ -166,7 +168,7 @@ int pk_digest_descriptors(pk_ctx *ctx, const uint8_t *enc_dev, uint64_t enc_byte
                           uint32_t D, uint8_t *digests_dev, int32_t *status_dev, pk_stream stream) {
     if (!ctx) return PK_ERR_ARG;
     if (D == 0) return PK_OK;
-    if (!enc_off_dev || !digests_dev || (enc_bytes && !enc_dev)) return PK_ERR_ARG;
+    if (!enc_off_dev || !digests_dev || (enc_bytes && !enc_dev) || !aligned(enc_off_dev, 8)) return PK_ERR_ARG;
     return cuda_rc(pk_launch_digest_descriptors(enc_dev, enc_bytes, enc_off_dev, D, digests_dev, status_dev,
                                                 reinterpret_cast<cudaStream_t>(stream)));
 }
@@ -181,6 +183,8 @@ int pk_derive_keys(pk_ctx *ctx, const int32_t *tokens_dev, uint64_t n_tokens, co
     if (key_capacity < n_tokens / ctx->chunk_tokens) return PK_ERR_ARG;
     if (key_capacity && (!keys_dev || !aligned16(keys_dev))) return PK_ERR_ARG;
     if (key_capacity > (uint64_t)0x7fffffff * 64) return PK_ERR_ARG;
+    if (!aligned(tokens_dev, 4) || !aligned(tok_off_dev, 8) || !aligned(desc_idx_dev, 4) || !aligned(key_off_dev, 8))
+        return PK_ERR_ARG;
     return cuda_rc(pk_launch_derive(ctx, tokens_dev, n_tokens, tok_off_dev, R, desc_idx_dev, digests_dev, D,
                                     key_off_dev, keys_dev, key_capacity, status_dev,
                                     reinterpret_cast<cudaStream_t>(stream)));
@@ -193,6 +197,7 @@ int pk_lookup(pk_ctx *ctx, const uint8_t *keys_dev, const int64_t *key_off_dev, 
     if (R && !hit_chunks_dev) return PK_ERR_ARG;
     if (key_capacity && (!keys_dev || !aligned16(keys_dev) || !slots_dev)) return PK_ERR_ARG;
     if (key_capacity > (uint64_t)0x7fffffff * 256) return PK_ERR_ARG;
+    if (!aligned(key_off_dev, 8) || !aligned(hit_chunks_dev, 4) || !aligned(slots_dev, 4)) return PK_ERR_ARG;
     return cuda_rc(pk_launch_lookup(ctx, keys_dev, key_off_dev, R, key_capacity, hit_chunks_dev, slots_dev,
                                     status_dev, reinterpret_cast<cudaStream_t>(stream)));
 }
@@ -205,6 +210,9 @@ int pk_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_dev, ui
     if (n == 0) return PK_OK;
     if (!keys_dev || !aligned16(keys_dev) || !slots_dev || !result_dev || !slot_out_dev) return PK_ERR_ARG;
     if (n > (uint64_t)0x7fffffff * 256 || n >= 0xffffffffull) return PK_ERR_ARG;
+    if (!aligned(slots_dev, 4) || !aligned(result_dev, 4) || !aligned(slot_out_dev, 4) || !aligned(key_off_dev, 8) ||
+        !aligned(hit_chunks_dev, 4))
+        return PK_ERR_ARG;
     const unsigned long long epoch = ++ctx->epoch;
     return cuda_rc(pk_launch_store(ctx, epoch, keys_dev, slots_dev, n, key_off_dev, hit_chunks_dev,
                                    key_off_dev ? R : 0, result_dev, slot_out_dev, status_dev,

@@ -16,13 +16,12 @@
 // that the result equals processing the entries one at a time in order.
 #include <cuda_runtime.h>
 
+#include "pk_device.cuh"
 #include "pk_internal.h"
 
 namespace {
 
-__device__ __forceinline__ void set_status(int32_t *status, int32_t code) {
-    if (status) atomicCAS(status, 0, code);
-}
+using pk::set_status;
 
 __device__ __forceinline__ bool is_zero(const uint4 &v) { return (v.x | v.y | v.z | v.w) == 0u; }
 __device__ __forceinline__ bool same(const uint4 &a, const uint4 &b) {
@@ -30,16 +29,6 @@ __device__ __forceinline__ bool same(const uint4 &a, const uint4 &b) {
 }
 __device__ __forceinline__ uint64_t home_of(const uint4 &k) {
     return ((uint64_t)k.y << 32) | k.x;  // bytes 0..7, little-endian
-}
-
-__device__ __forceinline__ uint32_t find_request(const int64_t *__restrict__ key_off, uint32_t R,
-                                                 int64_t g) {
-    uint32_t lo = 0, hi = R;  // key_off[lo] <= g < key_off[hi]
-    while (hi - lo > 1) {
-        const uint32_t mid = (lo + hi) >> 1;
-        if (__ldg(key_off + mid) <= g) lo = mid; else hi = mid;
-    }
-    return lo;
 }
 
 // Loads that observe concurrent writes of the same kernel.
@@ -59,17 +48,13 @@ __device__ __forceinline__ unsigned long long ld_volatile_u64(const unsigned lon
 // ---------------------------------------------------------------------------
 // Lookup
 // ---------------------------------------------------------------------------
-__global__ void k_hit_init(const int64_t *__restrict__ key_off, uint32_t R, int32_t *__restrict__ hit) {
-    const uint32_t r = blockIdx.x * blockDim.x + threadIdx.x;
-    if (r < R) hit[r] = (int32_t)(key_off[r + 1] - key_off[r]);
-}
-
+// One thread per key: slots[g] = the key's slot or PK_NO_SLOT.
 __global__ void __launch_bounds__(256)
 k_lookup(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
          const uint8_t *__restrict__ keys, const int64_t *__restrict__ key_off, uint32_t R,
-         int32_t *hit, uint32_t *__restrict__ slots, int32_t *status) {
+         uint64_t key_capacity, uint32_t *__restrict__ slots, int32_t *status) {
     const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (R == 0 || g >= __ldg(key_off + R)) return;
+    if (R == 0 || (uint64_t)g >= key_capacity || g >= __ldg(key_off + R)) return;
     const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * g));
     uint32_t slot = PK_NO_SLOT;
     if (!is_zero(key)) {
@@ -87,11 +72,32 @@ k_lookup(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
         if (s == max_probe) set_status(status, PK_ERR_PROBE_LIMIT);
     }
     slots[g] = slot;
-    if (slot == PK_NO_SLOT) {
-        const uint32_t r = find_request(key_off, R, g);
-        atomicMin(hit + r, (int32_t)(g - __ldg(key_off + r)));
-    }
 }
+
+// One warp per request: h_r = index of the first PK_NO_SLOT among its keys.
+__global__ void __launch_bounds__(256)
+k_first_miss(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capacity,
+             const uint32_t *__restrict__ slots, int32_t *__restrict__ hit) {
+    const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const uint32_t lane = threadIdx.x & 31;
+    if (r >= R) return;
+    const int64_t a = __ldg(key_off + r);
+    int64_t b = __ldg(key_off + r + 1);
+    if ((uint64_t)b > key_capacity) b = (int64_t)key_capacity;
+    int64_t h = b > a ? b - a : 0;
+    for (int64_t base = a; base < b; base += 32) {
+        const int64_t idx = base + lane;
+        const bool miss = idx < b && __ldg(slots + idx) == PK_NO_SLOT;
+        const uint32_t ball = __ballot_sync(0xffffffffu, miss);
+        if (ball) {
+            h = base - a + (__ffs(ball) - 1);
+            break;
+        }
+    }
+    if (lane == 0) hit[r] = (int32_t)h;
+}
+
+constexpr uint32_t kReserveAttempts = 64;
 
 // ---------------------------------------------------------------------------
 // Store, kernel 1 of 2: find or claim each key's entry.
@@ -108,20 +114,26 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
               const int32_t *__restrict__ hit, uint32_t R, int32_t *__restrict__ result,
               uint32_t *__restrict__ slot_out, int32_t *status) {
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (e >= n) return;
+    const uint64_t e0 = e - (threadIdx.x & 31);
+    if (e0 >= n) return;  // whole warp past the end
     if (key_off) {  // range mode: only [key_off[r] + hit[r], key_off[r+1])
         bool active = false;
-        if (R > 0 && (int64_t)e < __ldg(key_off + R)) {
-            const uint32_t r = find_request(key_off, R, (int64_t)e);
-            const int64_t h = __ldg(hit + r);
-            active = (int64_t)e - __ldg(key_off + r) >= (h > 0 ? h : 0);
+        const int64_t total = R > 0 ? __ldg(key_off + R) : 0;
+        if ((int64_t)e0 < total) {
+            const uint32_t r = pk::lane_request(key_off, R, (int64_t)e0, total, (int64_t)e);
+            if ((int64_t)e < total) {
+                const int64_t h = __ldg(hit + r);
+                active = (int64_t)e - __ldg(key_off + r) >= (h > 0 ? h : 0);
+            }
         }
+        if (e >= n) return;
         if (!active) {
             result[e] = PK_STORE_SKIPPED;
             slot_out[e] = PK_NO_SLOT;
             return;
         }
     }
+    if (e >= n) return;
     const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
     const uint32_t my_slot = slots[e];
     int32_t res = 0;
@@ -160,11 +172,27 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
                 break;
             }
             if (is_zero(v)) {
-                const unsigned long long c = atomicAdd(counter, 1ull);
-                if (c + 1ull >= capacity) {  // would leave no empty entry
+                // Reserve room for one more entry.  Threads that will lose the
+                // CAS below hold reservations briefly, so a refusal is retried
+                // (bounded, with backoff) after looking at the entry again.
+                bool reserved = false;
+                for (uint32_t attempt = 0; attempt < kReserveAttempts; ++attempt) {
+                    const unsigned long long c = atomicAdd(counter, 1ull);
+                    if (c + 1ull < capacity) {  // leaves at least one empty entry
+                        reserved = true;
+                        break;
+                    }
                     atomicAdd(counter, ~0ull);
-                    res = PK_ERR_TABLE_FULL;
-                    break;
+                    __nanosleep(64u << (attempt < 4 ? attempt : 4));
+                    v = ld_volatile_v4(ent->k);
+                    if (!is_zero(v)) break;
+                }
+                if (!reserved) {
+                    if (is_zero(v)) {
+                        res = PK_ERR_TABLE_FULL;
+                        break;
+                    }
+                    continue;  // the entry was taken meanwhile: examine it again
                 }
                 const uint4 old = atomicCAS(kp, make_uint4(0, 0, 0, 0), key);
                 if (is_zero(old)) {  // claimed
@@ -233,10 +261,10 @@ cudaError_t pk_launch_lookup(const pk_ctx *ctx, const uint8_t *keys, const int64
                              uint64_t key_capacity, int32_t *hit_chunks, uint32_t *slots, int32_t *status,
                              cudaStream_t s) {
     if (R == 0) return cudaSuccess;
-    k_hit_init<<<grid_for(R, 256), 256, 0, s>>>(key_off, R, hit_chunks);
     if (key_capacity > 0)
         k_lookup<<<grid_for(key_capacity, 256), 256, 0, s>>>(ctx->table, ctx->capacity - 1, ctx->max_probe, keys,
-                                                             key_off, R, hit_chunks, slots, status);
+                                                             key_off, R, key_capacity, slots, status);
+    k_first_miss<<<grid_for(32ull * R, 256), 256, 0, s>>>(key_off, R, key_capacity, slots, hit_chunks);
     return cudaGetLastError();
 }
 
