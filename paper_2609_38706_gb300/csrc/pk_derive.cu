@@ -22,19 +22,39 @@ namespace {
 using pk::set_status;
 
 // ---------------------------------------------------------------------------
-// Descriptor digests: one thread per descriptor.
+// Descriptor digests: one thread per descriptor.  The block's encodings are
+// first copied to shared memory with coalesced loads (when they fit), so the
+// byte-wise message assembly reads shared memory instead of global memory.
 // ---------------------------------------------------------------------------
-__global__ void k_digest_descriptors(const uint8_t *__restrict__ enc, uint64_t enc_bytes,
-                                     const int64_t *__restrict__ enc_off, uint32_t D,
-                                     uint8_t *__restrict__ digests, int32_t *status) {
-    const uint32_t j = blockIdx.x * blockDim.x + threadIdx.x;
-    if (j >= D) return;
+constexpr int kDescBlock = 64;
+constexpr int kDescStage = 32 * 1024;
+
+__global__ void __launch_bounds__(kDescBlock)
+k_digest_descriptors(const uint8_t *__restrict__ enc, uint64_t enc_bytes, const int64_t *__restrict__ enc_off,
+                     uint32_t D, uint8_t *__restrict__ digests, int32_t *status) {
+    __shared__ __align__(16) uint8_t stage[kDescStage];
+    __shared__ int64_t lo_s, hi_s;
+    const uint32_t j0 = blockIdx.x * kDescBlock;
+    const uint32_t j1 = min(D, j0 + kDescBlock);
+    if (threadIdx.x == 0) {
+        int64_t lo = enc_off[j0], hi = enc_off[j1];
+        if (lo < 0 || hi < lo || (uint64_t)hi > enc_bytes || hi - lo > kDescStage) lo = hi = -1;  // no staging
+        lo_s = lo;
+        hi_s = hi;
+    }
+    __syncthreads();
+    const int64_t lo = lo_s, hi = hi_s;
+    for (int64_t i = threadIdx.x; lo >= 0 && i < hi - lo; i += kDescBlock) stage[i] = enc[lo + i];
+    __syncthreads();
+    const uint32_t j = j0 + threadIdx.x;
+    if (j >= j1) return;
     const int64_t a = enc_off[j], b = enc_off[j + 1];
     if (a < 0 || b < a || (uint64_t)b > enc_bytes) {
         set_status(status, PK_ERR_ARG);
         return;
     }
-    pk::sha256_bytes(enc + a, (uint64_t)(b - a), digests + 32ull * j);
+    const bool staged = lo >= 0 && a >= lo && b <= hi;
+    pk::sha256_bytes(staged ? stage + (a - lo) : enc + a, (uint64_t)(b - a), digests + 32ull * j);
 }
 
 // ---------------------------------------------------------------------------
@@ -107,35 +127,53 @@ __device__ __forceinline__ void store_digest(uint8_t *dst, const uint32_t st[8])
 }
 
 // 16 message words of one 64-byte block of int32 tokens (little-endian bytes,
-// read by SHA-256 as big-endian words).
-__device__ __forceinline__ void load_block(const int32_t *__restrict__ src, bool aligned, uint32_t w[16]) {
-    if (aligned) {
-        const uint4 *q = reinterpret_cast<const uint4 *>(src);
+// read by SHA-256 as big-endian words), straight from global memory.
+__device__ __forceinline__ void load_block_global(const int32_t *__restrict__ src, uint32_t w[16]) {
 #pragma unroll
-        for (int v = 0; v < 4; ++v) {
-            const uint4 x = __ldg(q + v);
-            w[4 * v + 0] = pk::bswap32(x.x);
-            w[4 * v + 1] = pk::bswap32(x.y);
-            w[4 * v + 2] = pk::bswap32(x.z);
-            w[4 * v + 3] = pk::bswap32(x.w);
-        }
-    } else {
+    for (int t = 0; t < 16; ++t) w[t] = pk::bswap32((uint32_t)__ldg(src + t));
+}
+
+// Asynchronous 64-byte copy global -> shared (4 x 16 B; both 16-byte aligned).
+__device__ __forceinline__ void cp_async_block(uint32_t *smem_dst, const int32_t *src) {
+    const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
 #pragma unroll
-        for (int t = 0; t < 16; ++t) w[t] = pk::bswap32((uint32_t)__ldg(src + t));
+    for (int v = 0; v < 4; ++v)
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d + 16 * v), "l"(src + 4 * v) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Round constants and the padding block's schedule in shared memory.
+struct PadKW {
+    uint32_t kw[64];  // K_t + W_t of the final block of a message of 64k bytes (padding only)
+};
+
+__device__ __forceinline__ void load_tables(uint32_t *sK, uint32_t *sPad, const PadKW &pad) {
+    for (int i = threadIdx.x; i < 64; i += blockDim.x) {
+        sK[i] = pk::kSha256K[i];
+        sPad[i] = pad.kw[i];
     }
 }
 
 // ---------------------------------------------------------------------------
-// Chunk digests: one thread per chunk, 32 consecutive chunks per warp.  CT > 0
-// fixes the chunk size at compile time (the padding block is then a constant
-// message whose schedule the compiler folds); CT == 0 takes it at run time.
-// The next 64-byte block is loaded while the current one is compressed.
+// Chunk digests: one thread per chunk, 32 consecutive chunks per warp.  Token
+// blocks are staged through a 3-deep shared-memory ring with cp.async, so the
+// load of block b+2 overlaps the compression of block b.  For chunk sizes that
+// are multiples of 16 tokens the final block is pure padding, identical for
+// every chunk: it runs as rounds only on a schedule precomputed on the host.
 // ---------------------------------------------------------------------------
-template <int CT>
-__global__ void __launch_bounds__(128)
+constexpr int kDigestBlock = 128;
+constexpr int kStages = 3;
+
+__global__ void __launch_bounds__(kDigestBlock)
 k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_off,
-               const int64_t *__restrict__ key_off, uint32_t R, uint32_t C_rt,
+               const int64_t *__restrict__ key_off, uint32_t R, uint32_t C, const __grid_constant__ PadKW pad,
                uint8_t *__restrict__ keys) {
+    __shared__ uint32_t sK[64], sPad[64];
+    __shared__ __align__(16) uint32_t ring[kStages][kDigestBlock][16];
+    load_tables(sK, sPad, pad);
+    __syncthreads();
     if (R == 0) return;
     const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t g0 = g - (threadIdx.x & 31);
@@ -144,7 +182,6 @@ k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ t
     const uint32_t r = pk::lane_request(key_off, R, g0, total, g);
     if (g >= total) return;
     const int64_t i = g - __ldg(key_off + r);
-    const uint32_t C = CT > 0 ? (uint32_t)CT : C_rt;
     const int32_t *src = tokens + __ldg(tok_off + r) + i * (int64_t)C;
     const bool aligned = (reinterpret_cast<uintptr_t>(src) & 15) == 0;
 
@@ -152,20 +189,41 @@ k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ t
     pk::init_state(st);
     const uint32_t nfull = C / 16;
     uint32_t w[16];
-    if (nfull > 0) load_block(src, aligned, w);
-#pragma unroll 1
-    for (uint32_t b = 0; b < nfull; ++b) {
-        uint32_t nx[16];
-        if (b + 1 < nfull) load_block(src + 16 * (b + 1), aligned, nx);
-        pk::compress16(st, w);
+    if (aligned) {
 #pragma unroll
-        for (int t = 0; t < 16; ++t) w[t] = nx[t];
+        for (int b = 0; b < kStages - 1; ++b) {
+            if ((uint32_t)b < nfull) cp_async_block(ring[b][threadIdx.x], src + 16 * b);
+            cp_async_commit();
+        }
+#pragma unroll 1
+        for (uint32_t b = 0; b < nfull; ++b) {
+            const uint32_t ahead = b + kStages - 1;
+            if (ahead < nfull) cp_async_block(ring[ahead % kStages][threadIdx.x], src + 16 * ahead);
+            cp_async_commit();
+            cp_async_wait<kStages - 1>();  // block b has landed
+            const uint4 *q = reinterpret_cast<const uint4 *>(ring[b % kStages][threadIdx.x]);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+                const uint4 x = q[v];
+                w[4 * v + 0] = pk::bswap32(x.x);
+                w[4 * v + 1] = pk::bswap32(x.y);
+                w[4 * v + 2] = pk::bswap32(x.z);
+                w[4 * v + 3] = pk::bswap32(x.w);
+            }
+            pk::compress_rolled(st, w, sK);
+        }
+        cp_async_wait<0>();
+    } else {
+#pragma unroll 1
+        for (uint32_t b = 0; b < nfull; ++b) {
+            load_block_global(src + 16 * b, w);
+            pk::compress_rolled(st, w, sK);
+        }
     }
     const uint64_t bits = (uint64_t)C * 32u;
     const int rem = (int)(C % 16);
     if (rem == 0) {
-        pk::compress(st, 0x80000000u, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0,
-                     (uint32_t)(bits >> 32), (uint32_t)bits);
+        pk::compress_kw(st, sPad);
     } else {
         const int32_t *tail = src + 16 * nfull;
 #pragma unroll
@@ -174,11 +232,14 @@ k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ t
         if (rem <= 13) {
             w[14] = (uint32_t)(bits >> 32);
             w[15] = (uint32_t)bits;
-            pk::compress16(st, w);
+            pk::compress_rolled(st, w, sK);
         } else {
-            pk::compress16(st, w);
-            pk::compress(st, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0,
-                         (uint32_t)(bits >> 32), (uint32_t)bits);
+            pk::compress_rolled(st, w, sK);
+#pragma unroll
+            for (int t = 0; t < 16; ++t) w[t] = 0;
+            w[14] = (uint32_t)(bits >> 32);
+            w[15] = (uint32_t)bits;
+            pk::compress_rolled(st, w, sK);
         }
     }
     store_digest(keys + 32 * g, st);
@@ -186,11 +247,16 @@ k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ t
 
 // ---------------------------------------------------------------------------
 // Chain: one thread per request.  Message = k_{i-1} || d (block 1) then
-// c_i || padding for a 96-byte message (block 2, constant tail).
+// c_i || padding of a 96-byte message (block 2).
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(64)
+constexpr int kChainBlock = 32;
+
+__global__ void __launch_bounds__(kChainBlock)
 k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_idx,
         const uint8_t *__restrict__ digests, uint32_t R, uint32_t D, uint8_t *keys) {
+    __shared__ uint32_t sK[64];
+    for (int i = threadIdx.x; i < 64; i += blockDim.x) sK[i] = pk::kSha256K[i];
+    __syncthreads();
     const uint32_t r = blockIdx.x * blockDim.x + threadIdx.x;
     if (r >= R) return;
     const int64_t a = key_off[r];
@@ -200,9 +266,8 @@ k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_i
 
     const uint4 *dq = reinterpret_cast<const uint4 *>(digests + 32ull * di);
     const uint4 d_lo = __ldg(dq), d_hi = __ldg(dq + 1);
-    const uint32_t d0 = pk::bswap32(d_lo.x), d1 = pk::bswap32(d_lo.y), d2 = pk::bswap32(d_lo.z),
-                   d3 = pk::bswap32(d_lo.w), d4 = pk::bswap32(d_hi.x), d5 = pk::bswap32(d_hi.y),
-                   d6 = pk::bswap32(d_hi.z), d7 = pk::bswap32(d_hi.w);
+    const uint32_t dw[8] = {pk::bswap32(d_lo.x), pk::bswap32(d_lo.y), pk::bswap32(d_lo.z), pk::bswap32(d_lo.w),
+                            pk::bswap32(d_hi.x), pk::bswap32(d_hi.y), pk::bswap32(d_hi.z), pk::bswap32(d_hi.w)};
 
     uint4 *kq = reinterpret_cast<uint4 *>(keys + 32ull * a);
     uint32_t p[8] = {0, 0, 0, 0, 0, 0, 0, 0};  // k_{-1} = 0^32
@@ -216,10 +281,20 @@ k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_i
         }
         uint32_t st[8];
         pk::init_state(st);
-        pk::compress(st, p[0], p[1], p[2], p[3], p[4], p[5], p[6], p[7], d0, d1, d2, d3, d4, d5, d6, d7);
-        pk::compress(st, pk::bswap32(c_lo.x), pk::bswap32(c_lo.y), pk::bswap32(c_lo.z), pk::bswap32(c_lo.w),
-                     pk::bswap32(c_hi.x), pk::bswap32(c_hi.y), pk::bswap32(c_hi.z), pk::bswap32(c_hi.w),
-                     0x80000000u, 0, 0, 0, 0, 0, 0, 96u * 8u);
+        uint32_t w[16];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            w[j] = p[j];
+            w[8 + j] = dw[j];
+        }
+        pk::compress_rolled(st, w, sK);
+        w[0] = pk::bswap32(c_lo.x); w[1] = pk::bswap32(c_lo.y); w[2] = pk::bswap32(c_lo.z); w[3] = pk::bswap32(c_lo.w);
+        w[4] = pk::bswap32(c_hi.x); w[5] = pk::bswap32(c_hi.y); w[6] = pk::bswap32(c_hi.z); w[7] = pk::bswap32(c_hi.w);
+        w[8] = 0x80000000u;
+#pragma unroll
+        for (int j = 9; j < 15; ++j) w[j] = 0;
+        w[15] = 96u * 8u;
+        pk::compress_rolled(st, w, sK);
 #pragma unroll
         for (int j = 0; j < 8; ++j) p[j] = st[j];
         store_digest(keys + 32ull * (a + i), st);
@@ -235,7 +310,7 @@ unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1
 cudaError_t pk_launch_digest_descriptors(const uint8_t *enc, uint64_t enc_bytes, const int64_t *enc_off,
                                          uint32_t D, uint8_t *digests, int32_t *status, cudaStream_t s) {
     if (D == 0) return cudaSuccess;
-    k_digest_descriptors<<<grid_for(D, 64), 64, 0, s>>>(enc, enc_bytes, enc_off, D, digests, status);
+    k_digest_descriptors<<<grid_for(D, kDescBlock), kDescBlock, 0, s>>>(enc, enc_bytes, enc_off, D, digests, status);
     return cudaGetLastError();
 }
 
@@ -247,15 +322,10 @@ cudaError_t pk_launch_derive(const pk_ctx *ctx, const int32_t *tokens, uint64_t 
     k_chunk_offsets<<<1, kScanThreads, 0, s>>>(tok_off, R, n_tokens, C, desc_idx, D, key_capacity, key_off,
                                                status);
     if (R == 0 || key_capacity == 0) return cudaGetLastError();
-    constexpr unsigned kDigestBlock = 64;
-    const unsigned grid = grid_for(key_capacity, kDigestBlock);
-    if (C == 256)
-        k_chunk_digest<256><<<grid, kDigestBlock, 0, s>>>(tokens, tok_off, key_off, R, C, keys);
-    else if (C == 16)
-        k_chunk_digest<16><<<grid, kDigestBlock, 0, s>>>(tokens, tok_off, key_off, R, C, keys);
-    else
-        k_chunk_digest<0><<<grid, kDigestBlock, 0, s>>>(tokens, tok_off, key_off, R, C, keys);
-    constexpr unsigned kChainBlock = 32;
+    PadKW pad;
+    for (int t = 0; t < 64; ++t) pad.kw[t] = ctx->pad_kw[t];
+    k_chunk_digest<<<grid_for(key_capacity, kDigestBlock), kDigestBlock, 0, s>>>(tokens, tok_off, key_off, R, C, pad,
+                                                                                 keys);
     k_chain<<<grid_for(R, kChainBlock), kChainBlock, 0, s>>>(key_off, desc_idx, digests, R, D, keys);
     return cudaGetLastError();
 }

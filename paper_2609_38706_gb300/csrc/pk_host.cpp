@@ -107,6 +107,12 @@ int pk_init(pk_ctx **out, const pk_config *cfg, pk_stream stream) {
     c->max_probe = (cfg->max_probe == 0 || cfg->max_probe > c->capacity) ? (uint32_t)c->capacity : cfg->max_probe;
     c->table = static_cast<pk_entry *>(cfg->table_dev);
     c->epoch = 0;
+    {   // final block of a 4C-byte message when 4C is a multiple of 64: 0x80, zeros, 64-bit bit length
+        const uint64_t bits = (uint64_t)cfg->chunk_tokens * 32u;
+        const uint32_t m[16] = {0x80000000u, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, (uint32_t)(bits >> 32),
+                                (uint32_t)bits};
+        pk::kw_table(m, c->pad_kw);
+    }
     if (cudaMalloc(reinterpret_cast<void **>(&c->counter_dev), 256) != cudaSuccess) {
         delete c;
         return PK_ERR_CUDA;

@@ -27,6 +27,7 @@ struct pk_ctx {
     pk_entry *table;
     unsigned long long *counter_dev;  // number of entries in the table
     unsigned long long epoch;         // last store call number
+    uint32_t pad_kw[64];              // K_t + W_t of a chunk's final (padding-only) block, C % 16 == 0
 };
 
 // internal per-entry state between the two store kernels

@@ -193,3 +193,92 @@ PK_HD void sha256_bytes(const uint8_t *p, uint64_t len, uint8_t out[32]) {
 }
 
 }  // namespace pk
+
+#if defined(__CUDACC__)
+namespace pk {
+
+// Device-side compression with the 64 rounds written as a 16-round body that
+// is executed four times (the message schedule ring has period 16, and the
+// working-variable rotation period 8 divides 16, so one body serves all four
+// quarters).  Keeping the code a quarter of the fully unrolled size keeps a
+// loop of several compressions resident in the instruction cache; the round
+// constants are read from a shared-memory copy (sK, 64 words, see load_k).
+
+__device__ __forceinline__ void round_kw(uint32_t &a, uint32_t &b, uint32_t &c, uint32_t &d, uint32_t &e,
+                                         uint32_t &f, uint32_t &g, uint32_t &h, uint32_t kw) {
+    const uint32_t t1 = h + big_s1(e) + ch(e, f, g) + kw;
+    const uint32_t t2 = big_s0(a) + maj(a, b, c);
+    h = g; g = f; f = e; e = d + t1; d = c; c = b; b = a; a = t1 + t2;
+}
+
+template <bool SCHED>
+__device__ __forceinline__ void rounds16(uint32_t v[8], uint32_t w[16], const uint32_t *__restrict__ k16) {
+    uint32_t a = v[0], b = v[1], c = v[2], d = v[3], e = v[4], f = v[5], g = v[6], h = v[7];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        if (SCHED) w[j] += small_s1(w[(j + 14) & 15]) + w[(j + 9) & 15] + small_s0(w[(j + 1) & 15]);
+        round_kw(a, b, c, d, e, f, g, h, k16[j] + w[j]);
+    }
+    v[0] = a; v[1] = b; v[2] = c; v[3] = d; v[4] = e; v[5] = f; v[6] = g; v[7] = h;
+}
+
+// st <- st + compress(st, w); w is overwritten by the schedule.
+__device__ __forceinline__ void compress_rolled(uint32_t st[8], uint32_t w[16], const uint32_t *__restrict__ sK) {
+    uint32_t v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] = st[j];
+    rounds16<false>(v, w, sK);
+#pragma unroll 1
+    for (int q = 1; q < 4; ++q) rounds16<true>(v, w, sK + 16 * q);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) st[j] += v[j];
+}
+
+// st <- st + compress(st, W) for a message whose whole schedule is known in
+// advance: kw[t] = K_t + W_t for t = 0..63 (rounds only).
+__device__ __forceinline__ void compress_kw(uint32_t st[8], const uint32_t *__restrict__ kw) {
+    uint32_t a = st[0], b = st[1], c = st[2], d = st[3], e = st[4], f = st[5], g = st[6], h = st[7];
+#pragma unroll 1
+    for (int q = 0; q < 4; ++q) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) round_kw(a, b, c, d, e, f, g, h, kw[16 * q + j]);
+    }
+    st[0] += a; st[1] += b; st[2] += c; st[3] += d; st[4] += e; st[5] += f; st[6] += g; st[7] += h;
+}
+
+}  // namespace pk
+#endif
+
+namespace pk {
+
+// FIPS 180-4 round constants K_0..K_63 (section 4.2.2), as data for the
+// shared-memory copy used by the device compressions.
+#define PK_K_TABLE                                                                                   \
+    0x428a2f98u, 0x71374491u, 0xb5c0fbcfu, 0xe9b5dba5u, 0x3956c25bu, 0x59f111f1u, 0x923f82a4u,       \
+        0xab1c5ed5u, 0xd807aa98u, 0x12835b01u, 0x243185beu, 0x550c7dc3u, 0x72be5d74u, 0x80deb1feu,   \
+        0x9bdc06a7u, 0xc19bf174u, 0xe49b69c1u, 0xefbe4786u, 0x0fc19dc6u, 0x240ca1ccu, 0x2de92c6fu,   \
+        0x4a7484aau, 0x5cb0a9dcu, 0x76f988dau, 0x983e5152u, 0xa831c66du, 0xb00327c8u, 0xbf597fc7u,   \
+        0xc6e00bf3u, 0xd5a79147u, 0x06ca6351u, 0x14292967u, 0x27b70a85u, 0x2e1b2138u, 0x4d2c6dfcu,   \
+        0x53380d13u, 0x650a7354u, 0x766a0abbu, 0x81c2c92eu, 0x92722c85u, 0xa2bfe8a1u, 0xa81a664bu,   \
+        0xc24b8b70u, 0xc76c51a3u, 0xd192e819u, 0xd6990624u, 0xf40e3585u, 0x106aa070u, 0x19a4c116u,   \
+        0x1e376c08u, 0x2748774cu, 0x34b0bcb5u, 0x391c0cb3u, 0x4ed8aa4au, 0x5b9cca4fu, 0x682e6ff3u,   \
+        0x748f82eeu, 0x78a5636fu, 0x84c87814u, 0x8cc70208u, 0x90befffau, 0xa4506cebu, 0xbef9a3f7u,   \
+        0xc67178f2u
+
+#if defined(__CUDACC__)
+// Device copy of the round constants (one per translation unit), the source of
+// the shared-memory tables the compressions read.
+static __constant__ uint32_t kSha256K[64] = {PK_K_TABLE};
+#endif
+
+// Schedule-plus-constant table of a message block known on the host:
+// kw[t] = K_t + W_t (used for the constant final padding block of a chunk).
+PK_HD void kw_table(const uint32_t m[16], uint32_t kw[64]) {
+    const uint32_t K[64] = {PK_K_TABLE};
+    uint32_t W[64];
+    for (int t = 0; t < 16; ++t) W[t] = m[t];
+    for (int t = 16; t < 64; ++t) W[t] = small_s1(W[t - 2]) + W[t - 7] + small_s0(W[t - 15]) + W[t - 16];
+    for (int t = 0; t < 64; ++t) kw[t] = K[t] + W[t];
+}
+
+}  // namespace pk

@@ -45,6 +45,13 @@ __device__ __forceinline__ unsigned long long ld_volatile_u64(const unsigned lon
     return v;
 }
 
+// Entries are examined in windows of up to kWin consecutive entries (one
+// 128-byte line, aligned): the keys of a window are loaded together, so a
+// probe sequence costs one memory round trip per window instead of one per
+// entry.  The examination order is still home, home+1, ... as in plain
+// linear probing.
+constexpr uint32_t kWin = 4;
+
 // ---------------------------------------------------------------------------
 // Lookup
 // ---------------------------------------------------------------------------
@@ -58,18 +65,34 @@ k_lookup(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
     const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * g));
     uint32_t slot = PK_NO_SLOT;
     if (!is_zero(key)) {
-        const uint64_t home = home_of(key);
-        uint32_t s = 0;
-        for (; s < max_probe; ++s) {
-            const pk_entry *e = table + ((home + s) & mask);
-            const uint4 v = __ldg(reinterpret_cast<const uint4 *>(e->k));
-            if (same(v, key)) {
-                slot = __ldg(&e->slot);
-                break;
+        const uint32_t win = mask + 1 < kWin ? (uint32_t)(mask + 1) : kWin;
+        const uint64_t pos = home_of(key) & mask;
+        uint64_t base = pos & ~(uint64_t)(win - 1);
+        uint32_t j0 = (uint32_t)(pos - base);
+        uint32_t probed = 0;
+        bool done = false;
+        while (!done && probed < max_probe) {
+            const pk_entry *grp = table + base;
+            uint4 v[kWin];
+#pragma unroll
+            for (uint32_t u = 0; u < kWin; ++u)
+                if (u < win) v[u] = __ldg(reinterpret_cast<const uint4 *>(grp[u].k));
+#pragma unroll
+            for (uint32_t u = 0; u < kWin; ++u) {
+                if (u < win && u >= j0 && !done && probed < max_probe) {
+                    ++probed;
+                    if (same(v[u], key)) {
+                        slot = __ldg(&grp[u].slot);
+                        done = true;
+                    } else if (is_zero(v[u])) {
+                        done = true;
+                    }
+                }
             }
-            if (is_zero(v)) break;
+            base = (base + win) & mask;
+            j0 = 0;
         }
-        if (s == max_probe) set_status(status, PK_ERR_PROBE_LIMIT);
+        if (!done) set_status(status, PK_ERR_PROBE_LIMIT);
     }
     slots[g] = slot;
 }
@@ -97,16 +120,86 @@ k_first_miss(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capac
     if (lane == 0) hit[r] = (int32_t)h;
 }
 
-constexpr uint32_t kReserveAttempts = 64;
-
 // ---------------------------------------------------------------------------
 // Store, kernel 1 of 2: find or claim each key's entry.
 //   pre-existing key (epoch of an earlier call): PRESENT with its slot, final
-//   key absent: reserve capacity, CAS the key into the first empty entry
+//   key absent: CAS the key into the first empty entry
 //   key claimed in this call (by anyone): record the lowest claimant index in
 //   `owner` (atomicMax of ~index) and leave PENDING with the entry position
 //   in slot_out for kernel 2.
+// Capacity: when the table holds few enough entries that this call cannot
+// fill it (count + n < capacity), claims are counted once per warp at the
+// end; otherwise each claim first reserves room on the shared counter.
 // ---------------------------------------------------------------------------
+constexpr uint32_t kReserveAttempts = 64;
+
+enum Examine { kAdvance, kDone, kClaimedHere };
+
+// Examine entry `ent` (position pos) whose key was read as `cur`.
+__device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cur, const uint4 &key, uint32_t me,
+                                           unsigned long long epoch, bool fast, unsigned long long *counter,
+                                           uint64_t capacity, int32_t &res, uint32_t &out) {
+    uint4 *kp = reinterpret_cast<uint4 *>(ent->k);
+#pragma unroll 1
+    for (int pass = 0; pass < 2; ++pass) {
+        // A vector load racing a concurrent 128-bit CAS may observe a mix of
+        // zero and new words.  When every word is zero or equal to ours, take
+        // an atomic snapshot: a CAS that swaps our key for itself changes
+        // nothing and returns the entry's whole current key.
+        if (!same(cur, key) && !is_zero(cur) && (cur.x == 0 || cur.x == key.x) && (cur.y == 0 || cur.y == key.y) &&
+            (cur.z == 0 || cur.z == key.z) && (cur.w == 0 || cur.w == key.w))
+            cur = atomicCAS(kp, key, key);
+        if (same(cur, key)) {
+            const unsigned long long ep = ld_volatile_u64(&ent->epoch);
+            if (ep != 0ull && ep != epoch) {  // inserted by an earlier call
+                res = PK_STORE_PRESENT;
+                out = *(volatile uint32_t *)&ent->slot;
+            } else {  // claimed during this call
+                atomicMax(&ent->owner, me);
+                res = PK_STORE_PENDING;
+                out = (uint32_t)pos;
+            }
+            return kDone;
+        }
+        if (!is_zero(cur)) return kAdvance;  // a different key holds this entry
+        if (!fast) {
+            // Reserve room for one more entry.  Threads that will lose the CAS
+            // below hold reservations briefly, so a refusal is retried (bounded,
+            // with backoff) after looking at the entry again.
+            bool reserved = false;
+            for (uint32_t attempt = 0; attempt < kReserveAttempts; ++attempt) {
+                const unsigned long long c = atomicAdd(counter, 1ull);
+                if (c + 1ull < capacity) {  // leaves at least one empty entry
+                    reserved = true;
+                    break;
+                }
+                atomicAdd(counter, ~0ull);
+                __nanosleep(64u << (attempt < 4 ? attempt : 4));
+                cur = ld_volatile_v4(ent->k);
+                if (!is_zero(cur)) break;
+            }
+            if (!reserved) {
+                if (is_zero(cur)) {
+                    res = PK_ERR_TABLE_FULL;
+                    return kDone;
+                }
+                continue;  // the entry was taken meanwhile: examine it again
+            }
+        }
+        const uint4 old = atomicCAS(kp, make_uint4(0, 0, 0, 0), key);
+        if (is_zero(old)) {  // claimed
+            *(volatile unsigned long long *)&ent->epoch = epoch;
+            atomicMax(&ent->owner, me);
+            res = PK_STORE_PENDING;
+            out = (uint32_t)pos;
+            return fast ? kClaimedHere : kDone;
+        }
+        if (!fast) atomicAdd(counter, ~0ull);  // release the reservation
+        cur = old;                            // examine the winner's key
+    }
+    return kAdvance;
+}
+
 __global__ void __launch_bounds__(256)
 k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
               unsigned long long *counter, unsigned long long epoch, const uint8_t *__restrict__ keys,
@@ -114,108 +207,69 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
               const int32_t *__restrict__ hit, uint32_t R, int32_t *__restrict__ result,
               uint32_t *__restrict__ slot_out, int32_t *status) {
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const uint64_t e0 = e - (threadIdx.x & 31);
-    if (e0 >= n) return;  // whole warp past the end
+    const uint32_t lane = threadIdx.x & 31;
+    const uint64_t e0 = e - lane;
+    if (e0 >= n) return;  // whole warp past the end (uniform)
+    bool active = e < n;
     if (key_off) {  // range mode: only [key_off[r] + hit[r], key_off[r+1])
-        bool active = false;
         const int64_t total = R > 0 ? __ldg(key_off + R) : 0;
+        bool in_range = false;
         if ((int64_t)e0 < total) {
             const uint32_t r = pk::lane_request(key_off, R, (int64_t)e0, total, (int64_t)e);
             if ((int64_t)e < total) {
                 const int64_t h = __ldg(hit + r);
-                active = (int64_t)e - __ldg(key_off + r) >= (h > 0 ? h : 0);
+                in_range = (int64_t)e - __ldg(key_off + r) >= (h > 0 ? h : 0);
             }
         }
-        if (e >= n) return;
-        if (!active) {
-            result[e] = PK_STORE_SKIPPED;
-            slot_out[e] = PK_NO_SLOT;
-            return;
-        }
+        active = active && in_range;
     }
-    if (e >= n) return;
-    const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
-    const uint32_t my_slot = slots[e];
-    int32_t res = 0;
+    int32_t res = PK_STORE_SKIPPED;
     uint32_t out = PK_NO_SLOT;
-    if (is_zero(key)) {
-        res = PK_ERR_RESERVED_KEY;
-    } else if (my_slot == PK_NO_SLOT) {
-        res = PK_ERR_ARG;
-    } else {
-        const uint32_t me = ~(uint32_t)e;
-        const uint64_t home = home_of(key);
-        res = PK_ERR_PROBE_LIMIT;
-        uint32_t s = 0;
-        while (s < max_probe) {
-            const uint64_t pos = (home + s) & mask;
-            pk_entry *ent = table + pos;
-            uint4 *kp = reinterpret_cast<uint4 *>(ent->k);
-            uint4 v = ld_volatile_v4(ent->k);
-            // A vector load racing a concurrent 128-bit CAS may observe a mix of
-            // zero and new words.  When every word is zero or equal to ours, take
-            // an atomic snapshot instead: a CAS that swaps our key for itself
-            // changes nothing and returns the entry's whole current key.
-            if (!same(v, key) && !is_zero(v) && (v.x == 0 || v.x == key.x) && (v.y == 0 || v.y == key.y) &&
-                (v.z == 0 || v.z == key.z) && (v.w == 0 || v.w == key.w))
-                v = atomicCAS(kp, key, key);
-            if (same(v, key)) {
-                const unsigned long long ep = ld_volatile_u64(&ent->epoch);
-                if (ep != 0ull && ep != epoch) {  // inserted by an earlier call
-                    res = PK_STORE_PRESENT;
-                    out = *(volatile uint32_t *)&ent->slot;
-                } else {  // claimed during this call
-                    atomicMax(&ent->owner, me);
-                    res = PK_STORE_PENDING;
-                    out = (uint32_t)pos;
-                }
-                break;
-            }
-            if (is_zero(v)) {
-                // Reserve room for one more entry.  Threads that will lose the
-                // CAS below hold reservations briefly, so a refusal is retried
-                // (bounded, with backoff) after looking at the entry again.
-                bool reserved = false;
-                for (uint32_t attempt = 0; attempt < kReserveAttempts; ++attempt) {
-                    const unsigned long long c = atomicAdd(counter, 1ull);
-                    if (c + 1ull < capacity) {  // leaves at least one empty entry
-                        reserved = true;
-                        break;
+    bool claimed_fast = false;
+    if (active) {
+        const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
+        if (is_zero(key)) {
+            res = PK_ERR_RESERVED_KEY;
+        } else if (slots[e] == PK_NO_SLOT) {
+            res = PK_ERR_ARG;
+        } else {
+            const bool fast = ld_volatile_u64(counter) + n < capacity;
+            const uint32_t me = ~(uint32_t)e;
+            const uint32_t win = mask + 1 < kWin ? (uint32_t)(mask + 1) : kWin;
+            const uint64_t pos = home_of(key) & mask;
+            uint64_t base = pos & ~(uint64_t)(win - 1);
+            uint32_t j0 = (uint32_t)(pos - base);
+            uint32_t probed = 0;
+            bool done = false;
+            res = PK_ERR_PROBE_LIMIT;
+            while (!done && probed < max_probe) {
+                pk_entry *grp = table + base;
+                uint4 v[kWin];
+#pragma unroll
+                for (uint32_t u = 0; u < kWin; ++u)
+                    if (u < win) v[u] = ld_volatile_v4(grp[u].k);
+#pragma unroll
+                for (uint32_t u = 0; u < kWin; ++u) {
+                    if (u < win && u >= j0 && !done && probed < max_probe) {
+                        ++probed;
+                        const Examine x =
+                            examine(grp + u, base + u, v[u], key, me, epoch, fast, counter, capacity, res, out);
+                        if (x != kAdvance) done = true;
+                        if (x == kClaimedHere) claimed_fast = true;
                     }
-                    atomicAdd(counter, ~0ull);
-                    __nanosleep(64u << (attempt < 4 ? attempt : 4));
-                    v = ld_volatile_v4(ent->k);
-                    if (!is_zero(v)) break;
                 }
-                if (!reserved) {
-                    if (is_zero(v)) {
-                        res = PK_ERR_TABLE_FULL;
-                        break;
-                    }
-                    continue;  // the entry was taken meanwhile: examine it again
-                }
-                const uint4 old = atomicCAS(kp, make_uint4(0, 0, 0, 0), key);
-                if (is_zero(old)) {  // claimed
-                    *(volatile unsigned long long *)&ent->epoch = epoch;
-                    atomicMax(&ent->owner, me);
-                    res = PK_STORE_PENDING;
-                    out = (uint32_t)pos;
-                    break;
-                }
-                atomicAdd(counter, ~0ull);  // release the reservation
-                if (same(old, key)) {       // another entry of this call claimed it first
-                    atomicMax(&ent->owner, me);
-                    res = PK_STORE_PENDING;
-                    out = (uint32_t)pos;
-                    break;
-                }
+                base = (base + win) & mask;
+                j0 = 0;
             }
-            ++s;  // a different key holds this entry
         }
     }
-    result[e] = res;
-    slot_out[e] = out;
-    if (res < 0) set_status(status, res);
+    if (e < n) {
+        result[e] = res;
+        slot_out[e] = out;
+        if (res < 0) set_status(status, res);
+    }
+    const uint32_t m = __ballot_sync(0xffffffffu, claimed_fast);
+    if (lane == 0 && m) atomicAdd(counter, (unsigned long long)__popc(m));
 }
 
 // Store, kernel 2 of 2: the lowest claimant of each new key writes its slot.
