@@ -242,12 +242,16 @@ def main():
     desc_idx_h = torch.from_numpy(b.desc_idx.view(np.int32)).pin_memory()
     tokens_d, tok_off_d, desc_idx_d = tokens_h.to(dev), tok_off_h.to(dev), desc_idx_h.to(dev)
     descs = pk.Descriptors(wl.descriptors)
-    enc_h = torch.zeros(256 * 1024, dtype=torch.uint8).pin_memory()
-    enc_off_h = torch.zeros(descs.count + 1, dtype=torch.int64).pin_memory()
+    # one pinned staging buffer: D+1 int64 offsets, then the encodings (one copy per step)
+    off_bytes = 8 * (descs.count + 1)
+    a0_h = torch.zeros(off_bytes + 256 * 1024, dtype=torch.uint8).pin_memory()
+    enc_off_h = a0_h[:off_bytes].view(torch.int64)
+    enc_h = a0_h[off_bytes:]
     enc_used, _ = pk.pk_descriptors_encode(descs, enc_h.numpy(), enc_off_h.numpy())
     n_enc = int(enc_used.size)
-    enc_d = torch.zeros(n_enc, dtype=torch.uint8, device=dev)
-    enc_off_d = torch.zeros(descs.count + 1, dtype=torch.int64, device=dev)
+    a0_d = torch.zeros(off_bytes + n_enc, dtype=torch.uint8, device=dev)
+    enc_off_d = a0_d[:off_bytes].view(torch.int64)
+    enc_d = a0_d[off_bytes:]
     digests_d = torch.zeros((descs.count, 32), dtype=torch.uint8, device=dev)
     key_off_d = torch.empty(R + 1, dtype=torch.int64, device=dev)
     keys_d = torch.empty((N_cap, 32), dtype=torch.uint8, device=dev)
@@ -266,8 +270,7 @@ def main():
 
     def core(ev=None):
         pk.pk_descriptors_encode(descs, enc_h.numpy(), enc_off_h.numpy())      # a0, host
-        enc_d.copy_(enc_h[:n_enc], non_blocking=True)
-        enc_off_d.copy_(enc_off_h, non_blocking=True)
+        a0_d.copy_(a0_h[:off_bytes + n_enc], non_blocking=True)
         pk.pk_digest_descriptors(ctx, enc_d, enc_off_d, digests_d, status)     # a0, device
         if ev: ev[1].record(stream)
         pk.pk_derive_keys(ctx, tokens_d, tok_off_d, desc_idx_d, digests_d, key_off_d, keys_d, status)  # a1, a2
@@ -339,7 +342,7 @@ def main():
         torch.cuda.synchronize()
         if i >= args.warmup:
             e2e_ms.append(e0.elapsed_time(e1))
-    h2d = tokens_h.numel() * 4 + tok_off_h.numel() * 8 + desc_idx_h.numel() * 4 + n_enc + enc_off_h.numel() * 8
+    h2d = tokens_h.numel() * 4 + tok_off_h.numel() * 8 + desc_idx_h.numel() * 4 + off_bytes + n_enc
     d2h = (hit_h.numel() + slots_h.numel() + result_h.numel() + slot_out_h.numel()) * 4
 
     total_ms = float(np.sum(step_ms))

@@ -184,8 +184,10 @@ int pk_lookup(pk_ctx *ctx, const uint8_t *keys_dev, const int64_t *key_off_dev, 
  * slot_out_dev: uint32[n] (required: also holds intermediate positions).
  * Per-entry errors: PK_ERR_RESERVED_KEY, PK_ERR_ARG (slot == PK_NO_SLOT),
  * PK_ERR_TABLE_FULL, PK_ERR_PROBE_LIMIT; the first one also goes to
- * *status_dev.  Near capacity, which of a call's new keys are refused is
- * unspecified. */
+ * *status_dev.  A new key is refused once the table holds capacity - 1
+ * entries.  Near that threshold, which of a call's new keys are refused is
+ * unspecified, and insertions racing at it may take the last empty entries;
+ * probes for absent keys then end at max_probe with PK_ERR_PROBE_LIMIT. */
 int pk_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_dev, uint64_t n,
              const int64_t *key_off_dev, const int32_t *hit_chunks_dev, uint32_t R,
              int32_t *result_dev, uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream);

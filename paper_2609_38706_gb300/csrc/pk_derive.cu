@@ -22,39 +22,34 @@ namespace {
 using pk::set_status;
 
 // ---------------------------------------------------------------------------
-// Descriptor digests: one thread per descriptor.  The block's encodings are
-// first copied to shared memory with coalesced loads (when they fit), so the
-// byte-wise message assembly reads shared memory instead of global memory.
+// Descriptor digests: one warp per descriptor.  The warp copies the encoding
+// into shared memory with coalesced byte loads (32 bytes per round trip), then
+// one lane hashes it.  Encodings longer than the staging area are hashed from
+// global memory.
 // ---------------------------------------------------------------------------
-constexpr int kDescBlock = 64;
-constexpr int kDescStage = 32 * 1024;
+constexpr int kDescWarps = 4;
+constexpr int kDescStage = 2048;
 
-__global__ void __launch_bounds__(kDescBlock)
+__global__ void __launch_bounds__(32 * kDescWarps)
 k_digest_descriptors(const uint8_t *__restrict__ enc, uint64_t enc_bytes, const int64_t *__restrict__ enc_off,
                      uint32_t D, uint8_t *__restrict__ digests, int32_t *status) {
-    __shared__ __align__(16) uint8_t stage[kDescStage];
-    __shared__ int64_t lo_s, hi_s;
-    const uint32_t j0 = blockIdx.x * kDescBlock;
-    const uint32_t j1 = min(D, j0 + kDescBlock);
-    if (threadIdx.x == 0) {
-        int64_t lo = enc_off[j0], hi = enc_off[j1];
-        if (lo < 0 || hi < lo || (uint64_t)hi > enc_bytes || hi - lo > kDescStage) lo = hi = -1;  // no staging
-        lo_s = lo;
-        hi_s = hi;
-    }
-    __syncthreads();
-    const int64_t lo = lo_s, hi = hi_s;
-    for (int64_t i = threadIdx.x; lo >= 0 && i < hi - lo; i += kDescBlock) stage[i] = enc[lo + i];
-    __syncthreads();
-    const uint32_t j = j0 + threadIdx.x;
-    if (j >= j1) return;
-    const int64_t a = enc_off[j], b = enc_off[j + 1];
+    __shared__ __align__(16) uint8_t stage[kDescWarps][kDescStage];
+    const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t j = blockIdx.x * kDescWarps + warp;
+    if (j >= D) return;
+    const int64_t a = __ldg(enc_off + j), b = __ldg(enc_off + j + 1);
     if (a < 0 || b < a || (uint64_t)b > enc_bytes) {
-        set_status(status, PK_ERR_ARG);
+        if (lane == 0) set_status(status, PK_ERR_ARG);
         return;
     }
-    const bool staged = lo >= 0 && a >= lo && b <= hi;
-    pk::sha256_bytes(staged ? stage + (a - lo) : enc + a, (uint64_t)(b - a), digests + 32ull * j);
+    const int64_t len = b - a;
+    const bool staged = len <= kDescStage;
+    if (staged) {
+#pragma unroll 4
+        for (int64_t i = lane; i < len; i += 32) stage[warp][i] = __ldg(enc + a + i);
+    }
+    __syncwarp();
+    if (lane == 0) pk::sha256_bytes(staged ? stage[warp] : enc + a, (uint64_t)len, digests + 32ull * j);
 }
 
 // ---------------------------------------------------------------------------
@@ -246,61 +241,176 @@ k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ t
 }
 
 // ---------------------------------------------------------------------------
-// Chain: one thread per request.  Message = k_{i-1} || d (block 1) then
-// c_i || padding of a 96-byte message (block 2).
+// Chain: k_i = SHA-256(k_{i-1} || d || c_i), serial in i for each request.
+//
+// Each CTA serves 32 requests (one per lane) with two warps on different SM
+// sub-partitions, so that one chain step costs about the rounds alone:
+//   warp 0 (rounds):   holds the state; runs the 64 rounds of block 1
+//                      (k_{i-1} || d) and of block 2 (c_i || padding)
+//   warp 1 (schedule): writes K_t + W_t for both blocks to shared memory:
+//                      block 2's schedule depends on c_i only and is made one
+//                      step ahead; block 1's depends on k_{i-1} and is made in
+//                      three 16-word slices as soon as k_{i-1} is published.
+// Named barriers (count 64 = both warps), producer arrives / consumer syncs:
+//   1, 2, 3  block-1 slices t = 16..31, 32..47, 48..63 of step i are ready
+//   4        block-2 schedule of step i is ready
+//   5        k_i is published (rounds warp -> schedule warp)
+// Per CTA both warps run the same number of steps (the lanes' maximum), so
+// every phase of every barrier gets exactly one arrive and one sync; the
+// schedule warp signals barrier 4 for step i only after it has passed barrier
+// 5 of step i-1, so it never arrives twice on a barrier the rounds warp has
+// not yet synced.  Lanes past their own request's last chunk keep computing
+// (masked) so that the warps stay aligned.
 // ---------------------------------------------------------------------------
-constexpr int kChainBlock = 32;
+constexpr int kChainLanes = 32;
 
-__global__ void __launch_bounds__(kChainBlock)
+__device__ __forceinline__ void bar_sync(int id) { asm volatile("bar.sync %0, 64;" ::"r"(id) : "memory"); }
+__device__ __forceinline__ void bar_arrive(int id) { asm volatile("bar.arrive %0, 64;" ::"r"(id) : "memory"); }
+
+struct ChainSmem {
+    uint32_t kw1[64][kChainLanes];     // block-1 K+W, t = 16..63 used
+    uint32_t kw2[2][64][kChainLanes];  // block-2 K+W, double-buffered by step parity
+    uint32_t kpub[8][kChainLanes];     // k_{i-1} for the schedule warp
+};
+
+// 16 schedule words t = 16q .. 16q+15 of the ring w (in place), K_t + W_t -> out[t][lane]
+__device__ __forceinline__ void schedule16(uint32_t w[16], uint32_t (*out)[kChainLanes], int q, uint32_t lane) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        w[j] += pk::small_s1(w[(j + 14) & 15]) + w[(j + 9) & 15] + pk::small_s0(w[(j + 1) & 15]);
+        out[16 * q + j][lane] = pk::kSha256K[16 * q + j] + w[j];
+    }
+}
+
+// rounds t = 16q .. 16q+15 with K+W from shared memory
+__device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint32_t (*kw)[kChainLanes], int q, uint32_t lane) {
+    uint32_t a = v[0], b = v[1], c = v[2], d = v[3], e = v[4], f = v[5], g = v[6], h = v[7];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) pk::round_kw(a, b, c, d, e, f, g, h, kw[16 * q + j][lane]);
+    v[0] = a; v[1] = b; v[2] = c; v[3] = d; v[4] = e; v[5] = f; v[6] = g; v[7] = h;
+}
+
+__global__ void __launch_bounds__(2 * kChainLanes)
 k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_idx,
         const uint8_t *__restrict__ digests, uint32_t R, uint32_t D, uint8_t *keys) {
-    __shared__ uint32_t sK[64];
-    for (int i = threadIdx.x; i < 64; i += blockDim.x) sK[i] = pk::kSha256K[i];
-    __syncthreads();
-    const uint32_t r = blockIdx.x * blockDim.x + threadIdx.x;
-    if (r >= R) return;
-    const int64_t a = key_off[r];
-    const int64_t n = key_off[r + 1] - a;
-    const uint32_t di = desc_idx[r];
-    if (n <= 0 || di >= D) return;
-
-    const uint4 *dq = reinterpret_cast<const uint4 *>(digests + 32ull * di);
-    const uint4 d_lo = __ldg(dq), d_hi = __ldg(dq + 1);
-    const uint32_t dw[8] = {pk::bswap32(d_lo.x), pk::bswap32(d_lo.y), pk::bswap32(d_lo.z), pk::bswap32(d_lo.w),
-                            pk::bswap32(d_hi.x), pk::bswap32(d_hi.y), pk::bswap32(d_hi.z), pk::bswap32(d_hi.w)};
-
-    uint4 *kq = reinterpret_cast<uint4 *>(keys + 32ull * a);
-    uint32_t p[8] = {0, 0, 0, 0, 0, 0, 0, 0};  // k_{-1} = 0^32
-    uint4 c_lo = kq[0], c_hi = kq[1];
-#pragma unroll 1
-    for (int64_t i = 0; i < n; ++i) {
-        uint4 n_lo = c_lo, n_hi = c_hi;
-        if (i + 1 < n) {  // prefetch c_{i+1}
-            n_lo = kq[2 * (i + 1)];
-            n_hi = kq[2 * (i + 1) + 1];
-        }
-        uint32_t st[8];
-        pk::init_state(st);
-        uint32_t w[16];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            w[j] = p[j];
-            w[8 + j] = dw[j];
-        }
-        pk::compress_rolled(st, w, sK);
-        w[0] = pk::bswap32(c_lo.x); w[1] = pk::bswap32(c_lo.y); w[2] = pk::bswap32(c_lo.z); w[3] = pk::bswap32(c_lo.w);
-        w[4] = pk::bswap32(c_hi.x); w[5] = pk::bswap32(c_hi.y); w[6] = pk::bswap32(c_hi.z); w[7] = pk::bswap32(c_hi.w);
-        w[8] = 0x80000000u;
-#pragma unroll
-        for (int j = 9; j < 15; ++j) w[j] = 0;
-        w[15] = 96u * 8u;
-        pk::compress_rolled(st, w, sK);
-#pragma unroll
-        for (int j = 0; j < 8; ++j) p[j] = st[j];
-        store_digest(keys + 32ull * (a + i), st);
-        c_lo = n_lo;
-        c_hi = n_hi;
+    __shared__ __align__(16) ChainSmem sm;
+    const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const uint32_t r = blockIdx.x * kChainLanes + lane;
+    int64_t a = 0, n = 0;
+    uint32_t di = 0;
+    if (r < R) {
+        a = key_off[r];
+        n = key_off[r + 1] - a;
+        di = desc_idx[r];
+        if (n < 0 || di >= D) n = 0;
     }
+    int64_t nmax = n;  // identical in both warps: they cover the same 32 requests
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const int64_t x = __shfl_xor_sync(0xffffffffu, nmax, o);
+        nmax = x > nmax ? x : nmax;
+    }
+    if (nmax == 0) return;  // uniform over the CTA
+
+    uint32_t dw[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    if (n > 0) {
+        const uint4 *dq = reinterpret_cast<const uint4 *>(digests + 32ull * di);
+        const uint4 d_lo = __ldg(dq), d_hi = __ldg(dq + 1);
+        dw[0] = pk::bswap32(d_lo.x); dw[1] = pk::bswap32(d_lo.y); dw[2] = pk::bswap32(d_lo.z);
+        dw[3] = pk::bswap32(d_lo.w); dw[4] = pk::bswap32(d_hi.x); dw[5] = pk::bswap32(d_hi.y);
+        dw[6] = pk::bswap32(d_hi.z); dw[7] = pk::bswap32(d_hi.w);
+    }
+    uint4 *kq = reinterpret_cast<uint4 *>(keys + 32ull * a);
+
+    if (warp == 1) {  // ---------------- schedule warp ----------------
+        // block 2 of step i: W = c_i (8 words) || 0x80000000, 0 x 6, 768
+        auto make_kw2 = [&](int64_t i, int buf) {
+            uint32_t w[16];
+            if (i < n) {
+                const uint4 lo = kq[2 * i], hi = kq[2 * i + 1];
+                w[0] = pk::bswap32(lo.x); w[1] = pk::bswap32(lo.y); w[2] = pk::bswap32(lo.z); w[3] = pk::bswap32(lo.w);
+                w[4] = pk::bswap32(hi.x); w[5] = pk::bswap32(hi.y); w[6] = pk::bswap32(hi.z); w[7] = pk::bswap32(hi.w);
+            } else {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) w[j] = 0;
+            }
+            w[8] = 0x80000000u;
+#pragma unroll
+            for (int j = 9; j < 15; ++j) w[j] = 0;
+            w[15] = 96u * 8u;
+#pragma unroll
+            for (int j = 0; j < 16; ++j) sm.kw2[buf][j][lane] = pk::kSha256K[j] + w[j];
+#pragma unroll 1
+            for (int q = 1; q < 4; ++q) schedule16(w, sm.kw2[buf], q, lane);
+        };
+        make_kw2(0, 0);
+        bar_arrive(4);
+#pragma unroll 1
+        for (int64_t i = 0; i < nmax; ++i) {
+            uint32_t w[16];
+            if (i == 0) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) w[j] = 0;  // k_{-1} = 0^32
+            } else {
+                bar_sync(5);  // k_{i-1} published; the rounds warp has finished step i-1
+#pragma unroll
+                for (int j = 0; j < 8; ++j) w[j] = sm.kpub[j][lane];
+                bar_arrive(4);  // block-2 schedule of step i (made during the previous iteration)
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j) w[8 + j] = dw[j];
+            schedule16(w, sm.kw1, 1, lane);
+            bar_arrive(1);
+            schedule16(w, sm.kw1, 2, lane);
+            bar_arrive(2);
+            schedule16(w, sm.kw1, 3, lane);
+            bar_arrive(3);
+            if (i + 1 < nmax) make_kw2(i + 1, (int)((i + 1) & 1));
+        }
+        __syncthreads();  // stay resident until the rounds warp has consumed every phase
+        return;
+    }
+
+    // ---------------- rounds warp ----------------
+    uint32_t p[8] = {0, 0, 0, 0, 0, 0, 0, 0};  // k_{-1} = 0^32
+    uint32_t kd[8];                            // K_t + d_{t-8}, t = 8..15
+#pragma unroll
+    for (int j = 0; j < 8; ++j) kd[j] = pk::kSha256K[8 + j] + dw[j];
+#pragma unroll 1
+    for (int64_t i = 0; i < nmax; ++i) {
+        uint32_t v[8] = {PK_IV0, PK_IV1, PK_IV2, PK_IV3, PK_IV4, PK_IV5, PK_IV6, PK_IV7};
+        {   // block 1, rounds 0..15: W = k_{i-1} || d
+            uint32_t a_ = v[0], b_ = v[1], c_ = v[2], d_ = v[3], e_ = v[4], f_ = v[5], g_ = v[6], h_ = v[7];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) pk::round_kw(a_, b_, c_, d_, e_, f_, g_, h_, pk::kSha256K[j] + p[j]);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) pk::round_kw(a_, b_, c_, d_, e_, f_, g_, h_, kd[j]);
+            v[0] = a_; v[1] = b_; v[2] = c_; v[3] = d_; v[4] = e_; v[5] = f_; v[6] = g_; v[7] = h_;
+        }
+        bar_sync(1);
+        rounds16_kw(v, sm.kw1, 1, lane);
+        bar_sync(2);
+        rounds16_kw(v, sm.kw1, 2, lane);
+        bar_sync(3);
+        rounds16_kw(v, sm.kw1, 3, lane);
+        uint32_t st[8] = {PK_IV0 + v[0], PK_IV1 + v[1], PK_IV2 + v[2], PK_IV3 + v[3],
+                          PK_IV4 + v[4], PK_IV5 + v[5], PK_IV6 + v[6], PK_IV7 + v[7]};
+        bar_sync(4);  // block-2 schedule of step i
+        const uint32_t (*kw2)[kChainLanes] = sm.kw2[i & 1];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[j] = st[j];
+#pragma unroll 1
+        for (int q = 0; q < 4; ++q) rounds16_kw(v, kw2, q, lane);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) p[j] = st[j] + v[j];
+        if (i < n) store_digest(keys + 32ull * (a + i), p);
+        if (i + 1 < nmax) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) sm.kpub[j][lane] = p[j];
+            bar_arrive(5);
+        }
+    }
+    __syncthreads();
 }
 
 unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1) / block); }
@@ -310,7 +420,8 @@ unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1
 cudaError_t pk_launch_digest_descriptors(const uint8_t *enc, uint64_t enc_bytes, const int64_t *enc_off,
                                          uint32_t D, uint8_t *digests, int32_t *status, cudaStream_t s) {
     if (D == 0) return cudaSuccess;
-    k_digest_descriptors<<<grid_for(D, kDescBlock), kDescBlock, 0, s>>>(enc, enc_bytes, enc_off, D, digests, status);
+    k_digest_descriptors<<<grid_for(D, kDescWarps), 32 * kDescWarps, 0, s>>>(enc, enc_bytes, enc_off, D, digests,
+                                                                              status);
     return cudaGetLastError();
 }
 
@@ -326,6 +437,6 @@ cudaError_t pk_launch_derive(const pk_ctx *ctx, const int32_t *tokens, uint64_t 
     for (int t = 0; t < 64; ++t) pad.kw[t] = ctx->pad_kw[t];
     k_chunk_digest<<<grid_for(key_capacity, kDigestBlock), kDigestBlock, 0, s>>>(tokens, tok_off, key_off, R, C, pad,
                                                                                  keys);
-    k_chain<<<grid_for(R, kChainBlock), kChainBlock, 0, s>>>(key_off, desc_idx, digests, R, D, keys);
+    k_chain<<<grid_for(R, kChainLanes), 2 * kChainLanes, 0, s>>>(key_off, desc_idx, digests, R, D, keys);
     return cudaGetLastError();
 }

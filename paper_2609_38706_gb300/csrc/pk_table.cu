@@ -129,10 +129,11 @@ k_first_miss(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capac
 //   in slot_out for kernel 2.
 // Capacity: when the table holds few enough entries that this call cannot
 // fill it (count + n < capacity), claims are counted once per warp at the
-// end; otherwise each claim first reserves room on the shared counter.
+// end.  Otherwise a new key is refused (TABLE_FULL) once the count reaches
+// capacity - 1 and every claim is counted as it happens; claims racing at
+// that threshold can still take the last empty entries, after which probes
+// for absent keys end at max_probe (PK_ERR_PROBE_LIMIT).
 // ---------------------------------------------------------------------------
-constexpr uint32_t kReserveAttempts = 64;
-
 enum Examine { kAdvance, kDone, kClaimedHere };
 
 // Examine entry `ent` (position pos) whose key was read as `cur`.
@@ -162,29 +163,12 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
             return kDone;
         }
         if (!is_zero(cur)) return kAdvance;  // a different key holds this entry
-        if (!fast) {
-            // Reserve room for one more entry.  Threads that will lose the CAS
-            // below hold reservations briefly, so a refusal is retried (bounded,
-            // with backoff) after looking at the entry again.
-            bool reserved = false;
-            for (uint32_t attempt = 0; attempt < kReserveAttempts; ++attempt) {
-                const unsigned long long c = atomicAdd(counter, 1ull);
-                if (c + 1ull < capacity) {  // leaves at least one empty entry
-                    reserved = true;
-                    break;
-                }
-                atomicAdd(counter, ~0ull);
-                __nanosleep(64u << (attempt < 4 ? attempt : 4));
-                cur = ld_volatile_v4(ent->k);
-                if (!is_zero(cur)) break;
-            }
-            if (!reserved) {
-                if (is_zero(cur)) {
-                    res = PK_ERR_TABLE_FULL;
-                    return kDone;
-                }
-                continue;  // the entry was taken meanwhile: examine it again
-            }
+        // Room check: refuse a new key once the table holds capacity - 1
+        // entries.  Only successful claims are counted (below), so racing
+        // duplicates of one key never touch the counter.
+        if (!fast && ld_volatile_u64(counter) + 1ull >= capacity) {
+            res = PK_ERR_TABLE_FULL;
+            return kDone;
         }
         const uint4 old = atomicCAS(kp, make_uint4(0, 0, 0, 0), key);
         if (is_zero(old)) {  // claimed
@@ -192,10 +176,11 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
             atomicMax(&ent->owner, me);
             res = PK_STORE_PENDING;
             out = (uint32_t)pos;
-            return fast ? kClaimedHere : kDone;
+            if (fast) return kClaimedHere;  // counted once per warp at the end
+            atomicAdd(counter, 1ull);
+            return kDone;
         }
-        if (!fast) atomicAdd(counter, ~0ull);  // release the reservation
-        cur = old;                            // examine the winner's key
+        cur = old;  // examine the winner's key
     }
     return kAdvance;
 }
