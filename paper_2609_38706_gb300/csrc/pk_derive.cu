@@ -34,6 +34,8 @@ __global__ void __launch_bounds__(32 * kDescWarps)
 k_digest_descriptors(const uint8_t *__restrict__ enc, uint64_t enc_bytes, const int64_t *__restrict__ enc_off,
                      uint32_t D, uint8_t *__restrict__ digests, int32_t *status) {
     __shared__ __align__(16) uint8_t stage[kDescWarps][kDescStage];
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
     const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t j = blockIdx.x * kDescWarps + warp;
     if (j >= D) return;
@@ -64,6 +66,8 @@ k_chunk_offsets(const int64_t *__restrict__ tok_off, uint32_t R, uint64_t n_toke
                 int64_t *__restrict__ key_off, int32_t *status) {
     __shared__ long long warp_sums[kScanThreads / 32];
     __shared__ long long total_s;
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
     const uint32_t tid = threadIdx.x;
     const uint64_t per = (R + kScanThreads - 1) / kScanThreads;
     const uint64_t lo = tid * per;
@@ -167,8 +171,10 @@ k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ t
                uint8_t *__restrict__ keys) {
     __shared__ uint32_t sK[64], sPad[64];
     __shared__ __align__(16) uint32_t ring[kStages][kDigestBlock][16];
+    pk::pdl_launch_dependents();
     load_tables(sK, sPad, pad);
     __syncthreads();
+    pk::pdl_wait();
     if (R == 0) return;
     const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t g0 = g - (threadIdx.x & 31);
@@ -294,6 +300,8 @@ __global__ void __launch_bounds__(2 * kChainLanes)
 k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_idx,
         const uint8_t *__restrict__ digests, uint32_t R, uint32_t D, uint8_t *keys) {
     __shared__ __align__(16) ChainSmem sm;
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t r = blockIdx.x * kChainLanes + lane;
     int64_t a = 0, n = 0;
@@ -420,9 +428,10 @@ unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1
 cudaError_t pk_launch_digest_descriptors(const uint8_t *enc, uint64_t enc_bytes, const int64_t *enc_off,
                                          uint32_t D, uint8_t *digests, int32_t *status, cudaStream_t s) {
     if (D == 0) return cudaSuccess;
-    k_digest_descriptors<<<grid_for(D, kDescWarps), 32 * kDescWarps, 0, s>>>(enc, enc_bytes, enc_off, D, digests,
-                                                                              status);
-    return cudaGetLastError();
+    const cudaError_t e =
+        pk_launch(k_digest_descriptors, grid_for(D, kDescWarps), 32 * kDescWarps, s, enc, enc_bytes, enc_off, D,
+                  digests, status);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t pk_launch_derive(const pk_ctx *ctx, const int32_t *tokens, uint64_t n_tokens,
@@ -430,13 +439,16 @@ cudaError_t pk_launch_derive(const pk_ctx *ctx, const int32_t *tokens, uint64_t 
                              const uint8_t *digests, uint32_t D, int64_t *key_off, uint8_t *keys,
                              uint64_t key_capacity, int32_t *status, cudaStream_t s) {
     const uint32_t C = ctx->chunk_tokens;
-    k_chunk_offsets<<<1, kScanThreads, 0, s>>>(tok_off, R, n_tokens, C, desc_idx, D, key_capacity, key_off,
-                                               status);
-    if (R == 0 || key_capacity == 0) return cudaGetLastError();
+    cudaError_t e = pk_launch(k_chunk_offsets, 1, kScanThreads, s, tok_off, R, n_tokens, C, desc_idx, D, key_capacity,
+                              key_off, status);
+    if (e != cudaSuccess || R == 0 || key_capacity == 0) return e != cudaSuccess ? e : cudaGetLastError();
     PadKW pad;
     for (int t = 0; t < 64; ++t) pad.kw[t] = ctx->pad_kw[t];
-    k_chunk_digest<<<grid_for(key_capacity, kDigestBlock), kDigestBlock, 0, s>>>(tokens, tok_off, key_off, R, C, pad,
-                                                                                 keys);
-    k_chain<<<grid_for(R, kChainLanes), 2 * kChainLanes, 0, s>>>(key_off, desc_idx, digests, R, D, keys);
+    e = pk_launch(k_chunk_digest, grid_for(key_capacity, kDigestBlock), kDigestBlock, s, tokens, tok_off,
+                  (const int64_t *)key_off, R, C, pad, keys);
+    if (e != cudaSuccess) return e;
+    e = pk_launch(k_chain, grid_for(R, kChainLanes), 2 * kChainLanes, s, (const int64_t *)key_off, desc_idx, digests,
+                  R, D, keys);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

@@ -60,3 +60,15 @@ __device__ __forceinline__ uint32_t lane_request(const int64_t *__restrict__ key
 }
 
 }  // namespace pk
+
+namespace pk {
+
+// Programmatic dependent launch (sm_90+).  Every libpk kernel is launched with
+// programmatic stream serialization: it may become resident while the previous
+// kernel of the stream drains, lets its own successor do the same, and waits
+// for its predecessor's completion (and memory) before touching global memory.
+// Both are no-ops for a kernel launched without the attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+}  // namespace pk

@@ -48,3 +48,23 @@ cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const u
                             const uint32_t *slots, uint64_t n, const int64_t *key_off,
                             const int32_t *hit_chunks, uint32_t R, int32_t *result, uint32_t *slot_out,
                             int32_t *status, cudaStream_t s);
+
+#if defined(__CUDACC__)
+#include <utility>
+// Launch with programmatic stream serialization (see pk_device.cuh).
+template <typename... KArgs, typename... Args>
+static inline cudaError_t pk_launch(void (*kernel)(KArgs...), unsigned grid, unsigned block, cudaStream_t s,
+                                    Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(block);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+#endif

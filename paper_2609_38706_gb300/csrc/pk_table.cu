@@ -53,47 +53,87 @@ __device__ __forceinline__ unsigned long long ld_volatile_u64(const unsigned lon
 constexpr uint32_t kWin = 4;
 
 // ---------------------------------------------------------------------------
-// Lookup
+// Lookup of one key: its slot, or PK_NO_SLOT.  Returns false if the probe
+// sequence reached max_probe without an answer.
 // ---------------------------------------------------------------------------
-// One thread per key: slots[g] = the key's slot or PK_NO_SLOT.
+__device__ __forceinline__ bool probe(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
+                                      const uint4 &key, uint32_t &slot) {
+    slot = PK_NO_SLOT;
+    if (is_zero(key)) return true;  // the empty marker is never stored
+    const uint32_t win = mask + 1 < kWin ? (uint32_t)(mask + 1) : kWin;
+    const uint64_t pos = home_of(key) & mask;
+    uint64_t base = pos & ~(uint64_t)(win - 1);
+    uint32_t j0 = (uint32_t)(pos - base);
+    uint32_t probed = 0;
+    bool done = false;
+    while (!done && probed < max_probe) {
+        const pk_entry *grp = table + base;
+        uint4 v[kWin];
+#pragma unroll
+        for (uint32_t u = 0; u < kWin; ++u)
+            if (u < win) v[u] = __ldg(reinterpret_cast<const uint4 *>(grp[u].k));
+#pragma unroll
+        for (uint32_t u = 0; u < kWin; ++u) {
+            if (u < win && u >= j0 && !done && probed < max_probe) {
+                ++probed;
+                if (same(v[u], key)) {
+                    slot = __ldg(&grp[u].slot);
+                    done = true;
+                } else if (is_zero(v[u])) {
+                    done = true;
+                }
+            }
+        }
+        base = (base + win) & mask;
+        j0 = 0;
+    }
+    return done;
+}
+
+// One warp per request: every key's slot, and h_r = index of the first miss
+// (ballot over each group of 32 keys).  For batches of many short requests.
+__global__ void __launch_bounds__(256)
+k_lookup_req(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
+             const uint8_t *__restrict__ keys, const int64_t *__restrict__ key_off, uint32_t R,
+             uint64_t key_capacity, uint32_t *__restrict__ slots, int32_t *__restrict__ hit, int32_t *status) {
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
+    const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const uint32_t lane = threadIdx.x & 31;
+    if (r >= R) return;  // uniform per warp
+    const int64_t a = __ldg(key_off + r);
+    int64_t b = __ldg(key_off + r + 1);
+    if ((uint64_t)b > key_capacity) b = (int64_t)key_capacity;
+    int64_t h = -1;
+    bool limit = false;
+    for (int64_t base = a; base < b; base += 32) {
+        const int64_t g = base + lane;
+        uint32_t slot = PK_NO_SLOT;
+        if (g < b) {
+            const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * g));
+            if (!probe(table, mask, max_probe, key, slot)) limit = true;
+            slots[g] = slot;
+        }
+        const uint32_t ball = __ballot_sync(0xffffffffu, g < b && slot == PK_NO_SLOT);
+        if (h < 0 && ball) h = base - a + (__ffs(ball) - 1);
+    }
+    if (h < 0) h = b > a ? b - a : 0;
+    if (lane == 0) hit[r] = (int32_t)h;
+    if (limit) set_status(status, PK_ERR_PROBE_LIMIT);
+}
+
+// One thread per key (few long requests): slots only; k_first_miss follows.
 __global__ void __launch_bounds__(256)
 k_lookup(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
          const uint8_t *__restrict__ keys, const int64_t *__restrict__ key_off, uint32_t R,
          uint64_t key_capacity, uint32_t *__restrict__ slots, int32_t *status) {
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
     const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (R == 0 || (uint64_t)g >= key_capacity || g >= __ldg(key_off + R)) return;
     const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * g));
-    uint32_t slot = PK_NO_SLOT;
-    if (!is_zero(key)) {
-        const uint32_t win = mask + 1 < kWin ? (uint32_t)(mask + 1) : kWin;
-        const uint64_t pos = home_of(key) & mask;
-        uint64_t base = pos & ~(uint64_t)(win - 1);
-        uint32_t j0 = (uint32_t)(pos - base);
-        uint32_t probed = 0;
-        bool done = false;
-        while (!done && probed < max_probe) {
-            const pk_entry *grp = table + base;
-            uint4 v[kWin];
-#pragma unroll
-            for (uint32_t u = 0; u < kWin; ++u)
-                if (u < win) v[u] = __ldg(reinterpret_cast<const uint4 *>(grp[u].k));
-#pragma unroll
-            for (uint32_t u = 0; u < kWin; ++u) {
-                if (u < win && u >= j0 && !done && probed < max_probe) {
-                    ++probed;
-                    if (same(v[u], key)) {
-                        slot = __ldg(&grp[u].slot);
-                        done = true;
-                    } else if (is_zero(v[u])) {
-                        done = true;
-                    }
-                }
-            }
-            base = (base + win) & mask;
-            j0 = 0;
-        }
-        if (!done) set_status(status, PK_ERR_PROBE_LIMIT);
-    }
+    uint32_t slot;
+    if (!probe(table, mask, max_probe, key, slot)) set_status(status, PK_ERR_PROBE_LIMIT);
     slots[g] = slot;
 }
 
@@ -101,6 +141,8 @@ k_lookup(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
 __global__ void __launch_bounds__(256)
 k_first_miss(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capacity,
              const uint32_t *__restrict__ slots, int32_t *__restrict__ hit) {
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
     const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t lane = threadIdx.x & 31;
     if (r >= R) return;
@@ -185,12 +227,59 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
     return kAdvance;
 }
 
+// Insert-if-absent of one entry (index e): result code, output slot/position,
+// and whether it claimed an entry that the caller must count (fast mode).
+__device__ __forceinline__ void claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
+                                      unsigned long long *counter, unsigned long long epoch, bool fast,
+                                      const uint4 &key, uint32_t my_slot, uint64_t e, int32_t &res, uint32_t &out,
+                                      bool &claimed_fast) {
+    out = PK_NO_SLOT;
+    claimed_fast = false;
+    if (is_zero(key)) {
+        res = PK_ERR_RESERVED_KEY;
+        return;
+    }
+    if (my_slot == PK_NO_SLOT) {
+        res = PK_ERR_ARG;
+        return;
+    }
+    const uint32_t me = ~(uint32_t)e;
+    const uint32_t win = mask + 1 < kWin ? (uint32_t)(mask + 1) : kWin;
+    const uint64_t pos = home_of(key) & mask;
+    uint64_t base = pos & ~(uint64_t)(win - 1);
+    uint32_t j0 = (uint32_t)(pos - base);
+    uint32_t probed = 0;
+    bool done = false;
+    res = PK_ERR_PROBE_LIMIT;
+    while (!done && probed < max_probe) {
+        pk_entry *grp = table + base;
+        uint4 v[kWin];
+#pragma unroll
+        for (uint32_t u = 0; u < kWin; ++u)
+            if (u < win) v[u] = ld_volatile_v4(grp[u].k);
+#pragma unroll
+        for (uint32_t u = 0; u < kWin; ++u) {
+            if (u < win && u >= j0 && !done && probed < max_probe) {
+                ++probed;
+                const Examine x = examine(grp + u, base + u, v[u], key, me, epoch, fast, counter, capacity, res, out);
+                if (x != kAdvance) done = true;
+                if (x == kClaimedHere) claimed_fast = true;
+            }
+        }
+        base = (base + win) & mask;
+        j0 = 0;
+    }
+}
+
+// List mode, or range mode for few long requests: one thread per entry.
 __global__ void __launch_bounds__(256)
 k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
               unsigned long long *counter, unsigned long long epoch, const uint8_t *__restrict__ keys,
               const uint32_t *__restrict__ slots, uint64_t n, const int64_t *__restrict__ key_off,
               const int32_t *__restrict__ hit, uint32_t R, int32_t *__restrict__ result,
               uint32_t *__restrict__ slot_out, int32_t *status) {
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const uint32_t lane = threadIdx.x & 31;
     const uint64_t e0 = e - lane;
@@ -208,45 +297,15 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
         }
         active = active && in_range;
     }
+    unsigned long long cnt = 0;
+    if (lane == 0) cnt = ld_volatile_u64(counter);
+    const bool fast = __shfl_sync(0xffffffffu, cnt, 0) + n < capacity;
     int32_t res = PK_STORE_SKIPPED;
     uint32_t out = PK_NO_SLOT;
     bool claimed_fast = false;
     if (active) {
         const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
-        if (is_zero(key)) {
-            res = PK_ERR_RESERVED_KEY;
-        } else if (slots[e] == PK_NO_SLOT) {
-            res = PK_ERR_ARG;
-        } else {
-            const bool fast = ld_volatile_u64(counter) + n < capacity;
-            const uint32_t me = ~(uint32_t)e;
-            const uint32_t win = mask + 1 < kWin ? (uint32_t)(mask + 1) : kWin;
-            const uint64_t pos = home_of(key) & mask;
-            uint64_t base = pos & ~(uint64_t)(win - 1);
-            uint32_t j0 = (uint32_t)(pos - base);
-            uint32_t probed = 0;
-            bool done = false;
-            res = PK_ERR_PROBE_LIMIT;
-            while (!done && probed < max_probe) {
-                pk_entry *grp = table + base;
-                uint4 v[kWin];
-#pragma unroll
-                for (uint32_t u = 0; u < kWin; ++u)
-                    if (u < win) v[u] = ld_volatile_v4(grp[u].k);
-#pragma unroll
-                for (uint32_t u = 0; u < kWin; ++u) {
-                    if (u < win && u >= j0 && !done && probed < max_probe) {
-                        ++probed;
-                        const Examine x =
-                            examine(grp + u, base + u, v[u], key, me, epoch, fast, counter, capacity, res, out);
-                        if (x != kAdvance) done = true;
-                        if (x == kClaimedHere) claimed_fast = true;
-                    }
-                }
-                base = (base + win) & mask;
-                j0 = 0;
-            }
-        }
+        claim(table, mask, max_probe, capacity, counter, epoch, fast, key, slots[e], e, res, out, claimed_fast);
     }
     if (e < n) {
         result[e] = res;
@@ -257,12 +316,65 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
     if (lane == 0 && m) atomicAdd(counter, (unsigned long long)__popc(m));
 }
 
+// Range mode for many short requests: one warp per request, no search.
+// Writes every entry of [key_off[r], key_off[r+1]); entries past key_off[R]
+// are marked by the finalize kernel.
+__global__ void __launch_bounds__(256)
+k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
+                  unsigned long long *counter, unsigned long long epoch, const uint8_t *__restrict__ keys,
+                  const uint32_t *__restrict__ slots, uint64_t n, const int64_t *__restrict__ key_off,
+                  const int32_t *__restrict__ hit, uint32_t R, int32_t *__restrict__ result,
+                  uint32_t *__restrict__ slot_out, int32_t *status) {
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
+    const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const uint32_t lane = threadIdx.x & 31;
+    if (r >= R) return;  // uniform per warp
+    const int64_t a = __ldg(key_off + r);
+    int64_t b = __ldg(key_off + r + 1);
+    if ((uint64_t)b > n) b = (int64_t)n;
+    const int64_t h0 = __ldg(hit + r);
+    const int64_t first = a + (h0 > 0 ? h0 : 0);
+    unsigned long long cnt = 0;
+    if (lane == 0) cnt = ld_volatile_u64(counter);
+    const bool fast = __shfl_sync(0xffffffffu, cnt, 0) + n < capacity;
+    uint32_t claimed = 0;
+    for (int64_t base = a; base < b; base += 32) {
+        const int64_t e = base + lane;
+        int32_t res = PK_STORE_SKIPPED;
+        uint32_t out = PK_NO_SLOT;
+        bool claimed_fast = false;
+        if (e < b && e >= first) {
+            const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
+            claim(table, mask, max_probe, capacity, counter, epoch, fast, key, slots[e], (uint64_t)e, res, out,
+                  claimed_fast);
+        }
+        if (e < b) {
+            result[e] = res;
+            slot_out[e] = out;
+            if (res < 0) set_status(status, res);
+        }
+        claimed += __popc(__ballot_sync(0xffffffffu, claimed_fast));
+    }
+    if (lane == 0 && claimed) atomicAdd(counter, (unsigned long long)claimed);
+}
+
 // Store, kernel 2 of 2: the lowest claimant of each new key writes its slot.
+// In range mode, entries past key_off[R] (not keys of this batch) are skipped.
 __global__ void __launch_bounds__(256)
 k_store_finalize(pk_entry *table, const uint32_t *__restrict__ slots, uint64_t n,
-                 int32_t *__restrict__ result, uint32_t *__restrict__ slot_out) {
+                 const int64_t *__restrict__ key_off, uint32_t R, int32_t *__restrict__ result,
+                 uint32_t *__restrict__ slot_out) {
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (e >= n || result[e] != PK_STORE_PENDING) return;
+    if (e >= n) return;
+    if (key_off && (int64_t)e >= (R > 0 ? __ldg(key_off + R) : 0)) {
+        result[e] = PK_STORE_SKIPPED;
+        slot_out[e] = PK_NO_SLOT;
+        return;
+    }
+    if (result[e] != PK_STORE_PENDING) return;
     pk_entry *ent = table + slot_out[e];
     const uint32_t winner = ~ent->owner;
     if (winner == (uint32_t)e) {
@@ -288,6 +400,11 @@ __global__ void k_mark_loaded(pk_entry *table, uint64_t capacity) {
 
 unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1) / block); }
 
+// Per-request kernels when the batch has many short requests; per-key kernels
+// when a few requests carry many keys each (a warp per request would then
+// walk them serially).
+bool per_request(uint32_t R, uint64_t key_capacity) { return R >= 1024 || key_capacity <= 64ull * R; }
+
 }  // namespace
 
 cudaError_t pk_launch_mark_loaded(const pk_ctx *ctx, cudaStream_t s) {
@@ -300,11 +417,20 @@ cudaError_t pk_launch_lookup(const pk_ctx *ctx, const uint8_t *keys, const int64
                              uint64_t key_capacity, int32_t *hit_chunks, uint32_t *slots, int32_t *status,
                              cudaStream_t s) {
     if (R == 0) return cudaSuccess;
-    if (key_capacity > 0)
-        k_lookup<<<grid_for(key_capacity, 256), 256, 0, s>>>(ctx->table, ctx->capacity - 1, ctx->max_probe, keys,
-                                                             key_off, R, key_capacity, slots, status);
-    k_first_miss<<<grid_for(32ull * R, 256), 256, 0, s>>>(key_off, R, key_capacity, slots, hit_chunks);
-    return cudaGetLastError();
+    const uint64_t mask = ctx->capacity - 1;
+    cudaError_t e;
+    if (per_request(R, key_capacity)) {
+        e = pk_launch(k_lookup_req, grid_for(32ull * R, 256), 256, s, (const pk_entry *)ctx->table, mask,
+                      ctx->max_probe, keys, key_off, R, key_capacity, slots, hit_chunks, status);
+    } else {
+        e = key_capacity == 0 ? cudaSuccess
+                              : pk_launch(k_lookup, grid_for(key_capacity, 256), 256, s, (const pk_entry *)ctx->table,
+                                          mask, ctx->max_probe, keys, key_off, R, key_capacity, slots, status);
+        if (e == cudaSuccess)
+            e = pk_launch(k_first_miss, grid_for(32ull * R, 256), 256, s, key_off, R, key_capacity,
+                          (const uint32_t *)slots, hit_chunks);
+    }
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const uint8_t *keys,
@@ -312,10 +438,17 @@ cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const u
                             const int32_t *hit_chunks, uint32_t R, int32_t *result, uint32_t *slot_out,
                             int32_t *status, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
-    const unsigned grid = grid_for(n, 256);
-    k_store_claim<<<grid, 256, 0, s>>>(ctx->table, ctx->capacity - 1, ctx->max_probe, ctx->capacity,
-                                       ctx->counter_dev, epoch, keys, slots, n, key_off, hit_chunks, R, result,
-                                       slot_out, status);
-    k_store_finalize<<<grid, 256, 0, s>>>(ctx->table, slots, n, result, slot_out);
-    return cudaGetLastError();
+    const uint64_t mask = ctx->capacity - 1;
+    cudaError_t e;
+    if (key_off && R > 0 && per_request(R, n)) {
+        e = pk_launch(k_store_claim_req, grid_for(32ull * R, 256), 256, s, ctx->table, mask, ctx->max_probe,
+                      ctx->capacity, ctx->counter_dev, epoch, keys, slots, n, key_off, hit_chunks, R, result,
+                      slot_out, status);
+    } else {
+        e = pk_launch(k_store_claim, grid_for(n, 256), 256, s, ctx->table, mask, ctx->max_probe, ctx->capacity,
+                      ctx->counter_dev, epoch, keys, slots, n, key_off, hit_chunks, R, result, slot_out, status);
+    }
+    if (e == cudaSuccess)
+        e = pk_launch(k_store_finalize, grid_for(n, 256), 256, s, ctx->table, slots, n, key_off, R, result, slot_out);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
