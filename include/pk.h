@@ -158,6 +158,18 @@ int pk_derive_keys(pk_ctx *ctx, const int32_t *tokens_dev, uint64_t n_tokens,
                    uint8_t *keys_dev, uint64_t key_capacity, int32_t *status_dev,
                    pk_stream stream);
 
+/* Device.  pk_digest_descriptors and pk_derive_keys in one call: the
+ * descriptor encodings (as for pk_digest_descriptors) are hashed inside the
+ * key-derivation launch, alongside the chunk digests that do not depend on
+ * them, and the digests d are also written to digests_dev (D*32 bytes,
+ * 16-byte aligned).  Other arguments, outputs and errors as pk_derive_keys;
+ * D may be 0 only when R is 0. */
+int pk_derive_keys_enc(pk_ctx *ctx, const int32_t *tokens_dev, uint64_t n_tokens,
+                       const int64_t *tok_off_dev, uint32_t R, const uint32_t *desc_idx_dev,
+                       const uint8_t *enc_dev, uint64_t enc_bytes, const int64_t *enc_off_dev,
+                       uint32_t D, uint8_t *digests_dev, int64_t *key_off_dev, uint8_t *keys_dev,
+                       uint64_t key_capacity, int32_t *status_dev, pk_stream stream);
+
 /* Device.  Probe the table for every key of a pk_derive_keys result.
  *   slots_dev       OUT uint32[key_capacity]: slot of key i, or PK_NO_SLOT
  *   hit_chunks_dev  OUT int32[R]: h_r = the largest j such that keys 0..j-1 of

@@ -30,15 +30,11 @@ using pk::set_status;
 constexpr int kDescWarps = 4;
 constexpr int kDescStage = 2048;
 
-__global__ void __launch_bounds__(32 * kDescWarps)
-k_digest_descriptors(const uint8_t *__restrict__ enc, uint64_t enc_bytes, const int64_t *__restrict__ enc_off,
-                     uint32_t D, uint8_t *__restrict__ digests, int32_t *status) {
-    __shared__ __align__(16) uint8_t stage[kDescWarps][kDescStage];
-    pk::pdl_launch_dependents();
-    pk::pdl_wait();
-    const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const uint32_t j = blockIdx.x * kDescWarps + warp;
-    if (j >= D) return;
+// Warp `warp` of the calling block hashes descriptor j (all 32 lanes call).
+__device__ __forceinline__ void hash_descriptor(uint8_t *stage, const uint8_t *__restrict__ enc, uint64_t enc_bytes,
+                                                const int64_t *__restrict__ enc_off, uint32_t j,
+                                                uint8_t *__restrict__ digests, int32_t *status) {
+    const uint32_t lane = threadIdx.x & 31;
     const int64_t a = __ldg(enc_off + j), b = __ldg(enc_off + j + 1);
     if (a < 0 || b < a || (uint64_t)b > enc_bytes) {
         if (lane == 0) set_status(status, PK_ERR_ARG);
@@ -48,10 +44,21 @@ k_digest_descriptors(const uint8_t *__restrict__ enc, uint64_t enc_bytes, const 
     const bool staged = len <= kDescStage;
     if (staged) {
 #pragma unroll 4
-        for (int64_t i = lane; i < len; i += 32) stage[warp][i] = __ldg(enc + a + i);
+        for (int64_t i = lane; i < len; i += 32) stage[i] = __ldg(enc + a + i);
     }
     __syncwarp();
-    if (lane == 0) pk::sha256_bytes(staged ? stage[warp] : enc + a, (uint64_t)len, digests + 32ull * j);
+    if (lane == 0) pk::sha256_bytes(staged ? stage : enc + a, (uint64_t)len, digests + 32ull * j);
+}
+
+__global__ void __launch_bounds__(32 * kDescWarps)
+k_digest_descriptors(const uint8_t *__restrict__ enc, uint64_t enc_bytes, const int64_t *__restrict__ enc_off,
+                     uint32_t D, uint8_t *__restrict__ digests, int32_t *status) {
+    __shared__ __align__(16) uint8_t stage[kDescWarps][kDescStage];
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
+    const uint32_t warp = threadIdx.x >> 5;
+    const uint32_t j = blockIdx.x * kDescWarps + warp;
+    if (j < D) hash_descriptor(stage[warp], enc, enc_bytes, enc_off, j, digests, status);
 }
 
 // ---------------------------------------------------------------------------
@@ -165,18 +172,38 @@ __device__ __forceinline__ void load_tables(uint32_t *sK, uint32_t *sPad, const 
 constexpr int kDigestBlock = 128;
 constexpr int kStages = 3;
 
+// Optional descriptor work for the same launch (fused a0): the first
+// desc_blocks blocks hash descriptor encodings instead, one warp each.
+struct DescWork {
+    const uint8_t *enc;
+    uint64_t enc_bytes;
+    const int64_t *enc_off;
+    uint32_t D;
+    uint8_t *digests;
+    int32_t *status;
+    uint32_t desc_blocks;
+};
+
 __global__ void __launch_bounds__(kDigestBlock)
 k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_off,
                const int64_t *__restrict__ key_off, uint32_t R, uint32_t C, const __grid_constant__ PadKW pad,
-               uint8_t *__restrict__ keys) {
+               uint8_t *__restrict__ keys, const __grid_constant__ DescWork dw) {
     __shared__ uint32_t sK[64], sPad[64];
     __shared__ __align__(16) uint32_t ring[kStages][kDigestBlock][16];
     pk::pdl_launch_dependents();
+    if (blockIdx.x < dw.desc_blocks) {
+        pk::pdl_wait();
+        const uint32_t warp = threadIdx.x >> 5;
+        const uint32_t j = blockIdx.x * (kDigestBlock / 32) + warp;
+        uint8_t *stage = reinterpret_cast<uint8_t *>(ring[0]) + warp * kDescStage;  // 4 x 2 KiB of the ring
+        if (j < dw.D) hash_descriptor(stage, dw.enc, dw.enc_bytes, dw.enc_off, j, dw.digests, dw.status);
+        return;
+    }
     load_tables(sK, sPad, pad);
     __syncthreads();
     pk::pdl_wait();
     if (R == 0) return;
-    const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t g = (int64_t)(blockIdx.x - dw.desc_blocks) * blockDim.x + threadIdx.x;
     const int64_t g0 = g - (threadIdx.x & 31);
     const int64_t total = __ldg(key_off + R);
     if (g0 >= total) return;  // whole warp past the end
@@ -438,17 +465,36 @@ cudaError_t pk_launch_derive(const pk_ctx *ctx, const int32_t *tokens, uint64_t 
                              const int64_t *tok_off, uint32_t R, const uint32_t *desc_idx,
                              const uint8_t *digests, uint32_t D, int64_t *key_off, uint8_t *keys,
                              uint64_t key_capacity, int32_t *status, cudaStream_t s) {
+    return pk_launch_derive_enc(ctx, tokens, n_tokens, tok_off, R, desc_idx, nullptr, 0, nullptr, D,
+                                const_cast<uint8_t *>(digests), key_off, keys, key_capacity, status, s);
+}
+
+cudaError_t pk_launch_derive_enc(const pk_ctx *ctx, const int32_t *tokens, uint64_t n_tokens,
+                                 const int64_t *tok_off, uint32_t R, const uint32_t *desc_idx, const uint8_t *enc,
+                                 uint64_t enc_bytes, const int64_t *enc_off, uint32_t D, uint8_t *digests,
+                                 int64_t *key_off, uint8_t *keys, uint64_t key_capacity, int32_t *status,
+                                 cudaStream_t s) {
+    static_assert(kDigestBlock / 32 * kDescStage <= (int)sizeof(uint32_t) * kStages * kDigestBlock * 16,
+                  "descriptor staging fits in the token ring");
     const uint32_t C = ctx->chunk_tokens;
     cudaError_t e = pk_launch(k_chunk_offsets, 1, kScanThreads, s, tok_off, R, n_tokens, C, desc_idx, D, key_capacity,
                               key_off, status);
-    if (e != cudaSuccess || R == 0 || key_capacity == 0) return e != cudaSuccess ? e : cudaGetLastError();
-    PadKW pad;
-    for (int t = 0; t < 64; ++t) pad.kw[t] = ctx->pad_kw[t];
-    e = pk_launch(k_chunk_digest, grid_for(key_capacity, kDigestBlock), kDigestBlock, s, tokens, tok_off,
-                  (const int64_t *)key_off, R, C, pad, keys);
     if (e != cudaSuccess) return e;
-    e = pk_launch(k_chain, grid_for(R, kChainLanes), 2 * kChainLanes, s, (const int64_t *)key_off, desc_idx, digests,
-                  R, D, keys);
-    if (e != cudaSuccess) return e;
+    DescWork dw = {enc, enc_bytes, enc_off, D, digests, status, 0};
+    if (enc_off) dw.desc_blocks = grid_for(D, kDigestBlock / 32);
+    const bool chunks = R > 0 && key_capacity > 0;
+    const unsigned digest_blocks = chunks ? grid_for(key_capacity, kDigestBlock) : 0;
+    if (digest_blocks + dw.desc_blocks > 0) {
+        PadKW pad;
+        for (int t = 0; t < 64; ++t) pad.kw[t] = ctx->pad_kw[t];
+        e = pk_launch(k_chunk_digest, digest_blocks + dw.desc_blocks, kDigestBlock, s, tokens, tok_off,
+                      (const int64_t *)key_off, R, C, pad, keys, dw);
+        if (e != cudaSuccess) return e;
+    }
+    if (chunks) {
+        e = pk_launch(k_chain, grid_for(R, kChainLanes), 2 * kChainLanes, s, (const int64_t *)key_off, desc_idx,
+                      (const uint8_t *)digests, R, D, keys);
+        if (e != cudaSuccess) return e;
+    }
     return cudaGetLastError();
 }

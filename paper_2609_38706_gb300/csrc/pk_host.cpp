@@ -196,6 +196,25 @@ int pk_derive_keys(pk_ctx *ctx, const int32_t *tokens_dev, uint64_t n_tokens, co
                                     reinterpret_cast<cudaStream_t>(stream)));
 }
 
+int pk_derive_keys_enc(pk_ctx *ctx, const int32_t *tokens_dev, uint64_t n_tokens, const int64_t *tok_off_dev,
+                       uint32_t R, const uint32_t *desc_idx_dev, const uint8_t *enc_dev, uint64_t enc_bytes,
+                       const int64_t *enc_off_dev, uint32_t D, uint8_t *digests_dev, int64_t *key_off_dev,
+                       uint8_t *keys_dev, uint64_t key_capacity, int32_t *status_dev, pk_stream stream) {
+    if (!ctx || !tok_off_dev || !key_off_dev) return PK_ERR_ARG;
+    if (n_tokens && !tokens_dev) return PK_ERR_ARG;
+    if (R && (!desc_idx_dev || D == 0)) return PK_ERR_ARG;
+    if (D && (!enc_off_dev || !digests_dev || !aligned16(digests_dev) || !aligned(enc_off_dev, 8))) return PK_ERR_ARG;
+    if (enc_bytes && !enc_dev) return PK_ERR_ARG;
+    if (key_capacity < n_tokens / ctx->chunk_tokens) return PK_ERR_ARG;
+    if (key_capacity && (!keys_dev || !aligned16(keys_dev))) return PK_ERR_ARG;
+    if (key_capacity > (uint64_t)0x7fffffff * 64) return PK_ERR_ARG;
+    if (!aligned(tokens_dev, 4) || !aligned(tok_off_dev, 8) || !aligned(desc_idx_dev, 4) || !aligned(key_off_dev, 8))
+        return PK_ERR_ARG;
+    return cuda_rc(pk_launch_derive_enc(ctx, tokens_dev, n_tokens, tok_off_dev, R, desc_idx_dev, enc_dev, enc_bytes,
+                                        D ? enc_off_dev : nullptr, D, digests_dev, key_off_dev, keys_dev,
+                                        key_capacity, status_dev, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 int pk_lookup(pk_ctx *ctx, const uint8_t *keys_dev, const int64_t *key_off_dev, uint32_t R,
               uint64_t key_capacity, int32_t *hit_chunks_dev, uint32_t *slots_dev, int32_t *status_dev,
               pk_stream stream) {

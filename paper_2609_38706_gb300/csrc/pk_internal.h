@@ -40,6 +40,11 @@ cudaError_t pk_launch_derive(const pk_ctx *ctx, const int32_t *tokens, uint64_t 
                              const int64_t *tok_off, uint32_t R, const uint32_t *desc_idx,
                              const uint8_t *digests, uint32_t D, int64_t *key_off, uint8_t *keys,
                              uint64_t key_capacity, int32_t *status, cudaStream_t s);
+cudaError_t pk_launch_derive_enc(const pk_ctx *ctx, const int32_t *tokens, uint64_t n_tokens,
+                                 const int64_t *tok_off, uint32_t R, const uint32_t *desc_idx, const uint8_t *enc,
+                                 uint64_t enc_bytes, const int64_t *enc_off, uint32_t D, uint8_t *digests,
+                                 int64_t *key_off, uint8_t *keys, uint64_t key_capacity, int32_t *status,
+                                 cudaStream_t s);
 cudaError_t pk_launch_lookup(const pk_ctx *ctx, const uint8_t *keys, const int64_t *key_off, uint32_t R,
                              uint64_t key_capacity, int32_t *hit_chunks, uint32_t *slots, int32_t *status,
                              cudaStream_t s);

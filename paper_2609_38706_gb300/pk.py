@@ -80,6 +80,8 @@ def lib() -> ctypes.CDLL:
             "pk_digest_descriptors": (ctypes.c_int, [_VP, _VP, _U64, _VP, _U32, _VP, _VP, _VP]),
             "pk_derive_keys": (ctypes.c_int, [_VP, _VP, _U64, _VP, _U32, _VP, _VP, _U32, _VP, _VP, _U64,
                                               _VP, _VP]),
+            "pk_derive_keys_enc": (ctypes.c_int, [_VP, _VP, _U64, _VP, _U32, _VP, _VP, _U64, _VP, _U32, _VP, _VP, _VP,
+                                                  _U64, _VP, _VP]),
             "pk_lookup": (ctypes.c_int, [_VP, _VP, _VP, _U32, _U64, _VP, _VP, _VP, _VP]),
             "pk_store": (ctypes.c_int, [_VP, _VP, _VP, _U64, _VP, _VP, _U32, _VP, _VP, _VP, _VP]),
             "pk_entries": (ctypes.c_int, [_VP, ctypes.POINTER(ctypes.c_uint64), _VP]),
@@ -229,6 +231,16 @@ def pk_derive_keys(ctx: int, tokens: torch.Tensor, tok_off: torch.Tensor, desc_i
     _check(lib().pk_derive_keys(ctx, _p(tokens), tokens.numel(), _p(tok_off), R, _p(desc_idx), _p(digests), D,
                                 _p(key_off), _p(keys), keys.numel() // 32, _p(status), _s(stream)),
            "pk_derive_keys")
+
+
+def pk_derive_keys_enc(ctx: int, tokens: torch.Tensor, tok_off: torch.Tensor, desc_idx: torch.Tensor,
+                       enc: torch.Tensor, enc_off: torch.Tensor, digests: torch.Tensor, key_off: torch.Tensor,
+                       keys: torch.Tensor, status: torch.Tensor, stream=None) -> None:
+    R = tok_off.numel() - 1
+    D = enc_off.numel() - 1
+    _check(lib().pk_derive_keys_enc(ctx, _p(tokens), tokens.numel(), _p(tok_off), R, _p(desc_idx), _p(enc),
+                                    enc.numel(), _p(enc_off), D, _p(digests), _p(key_off), _p(keys),
+                                    keys.numel() // 32, _p(status), _s(stream)), "pk_derive_keys_enc")
 
 
 def pk_lookup(ctx: int, keys: torch.Tensor, key_off: torch.Tensor, hit_chunks: torch.Tensor,

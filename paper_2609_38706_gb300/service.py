@@ -103,6 +103,24 @@ class KeyTable:
         pk.pk_derive_keys(self.ctx, tokens, tok_off, desc_idx, digests, key_off, keys, self.status, self.stream)
         return key_off, keys
 
+    def derive_enc(self, tokens, tok_off, desc_idx, descriptors):
+        """Descriptor digests and keys in one call (pk_derive_keys_enc)."""
+        enc, off = pk.pk_descriptors_encode(descriptors)
+        D = off.size - 1
+        enc_d = _dev(enc if enc.size else np.zeros(1, np.uint8), torch.uint8, self.device)[: enc.size]
+        off_d = _dev(off, torch.int64, self.device)
+        digests = torch.zeros((max(D, 1), 32), dtype=torch.uint8, device=self.device)[:D]
+        tokens = _dev(tokens, torch.int32, self.device)
+        tok_off = _dev(tok_off, torch.int64, self.device)
+        desc_idx = _dev(desc_idx, torch.int32, self.device)
+        R = tok_off.numel() - 1
+        cap = tokens.numel() // self.chunk_tokens
+        key_off = torch.empty(R + 1, dtype=torch.int64, device=self.device)
+        keys = torch.empty((max(cap, 0), 32), dtype=torch.uint8, device=self.device)
+        pk.pk_derive_keys_enc(self.ctx, tokens, tok_off, desc_idx, enc_d, off_d, digests, key_off, keys,
+                              self.status, self.stream)
+        return digests, key_off, keys
+
     def lookup(self, keys, key_off):
         R = key_off.numel() - 1
         hit = torch.empty(R, dtype=torch.int32, device=self.device)

@@ -114,6 +114,34 @@ def test_full_configs_every_key(name):
         assert len({bytes(x) for x in O.prefix128(g["prior_keys"])}) == 16 * D   # Sec. 6.5 storage growth
 
 
+@pytest.mark.parametrize("name", REDUCED)
+def test_fused_descriptor_and_key_derivation(name):
+    """pk_derive_keys_enc: digests d and keys from one launch sequence."""
+    from paper_2609_38706_gb300.service import KeyTable
+    wl = W.reduced(name)
+    b = wl.batch
+    kt = KeyTable(wl.chunk_tokens, wl.capacity_log2)
+    d, ko, keys = kt.derive_enc(b.tokens, b.tok_off, b.desc_idx, wl.descriptors)
+    kt.check("derive_enc")
+    rd = O.descriptor_digests(wl.descriptors)
+    rko, rkeys = O.derive_keys(b.tokens, b.tok_off, wl.chunk_tokens, b.desc_idx, rd)
+    assert np.array_equal(d.cpu().numpy(), rd)
+    assert np.array_equal(ko.cpu().numpy(), rko)
+    assert np.array_equal(keys.cpu().numpy()[: rkeys.shape[0]], rkeys)
+    kt.close()
+
+
+def test_fused_empty_batch():
+    from paper_2609_38706_gb300.service import KeyTable
+    kt = KeyTable(16, 6)
+    d, ko, keys = kt.derive_enc(np.zeros(0, np.int32), np.zeros(1, np.int64), np.zeros(0, np.uint32),
+                                [W.tiny().descriptors[0]])
+    kt.check()
+    assert ko.cpu().tolist() == [0] and keys.shape[0] == 0
+    assert d.cpu().numpy().tobytes() == O.descriptor_digest(W.tiny().descriptors[0])
+    kt.close()
+
+
 def test_cross_context_stability():
     """Two independent contexts (two 'workers') derive identical keys."""
     from paper_2609_38706_gb300.service import KeyTable
