@@ -278,17 +278,20 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
               const uint32_t *__restrict__ slots, uint64_t n, const int64_t *__restrict__ key_off,
               const int32_t *__restrict__ hit, uint32_t R, int32_t *__restrict__ result,
               uint32_t *__restrict__ slot_out, int32_t *status) {
+    // Claims are counted once per block: same-address atomics serialise in L2.
+    __shared__ unsigned long long block_claims;
+    if (threadIdx.x == 0) block_claims = 0;
+    __syncthreads();
     pk::pdl_launch_dependents();
     pk::pdl_wait();
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const uint32_t lane = threadIdx.x & 31;
     const uint64_t e0 = e - lane;
-    if (e0 >= n) return;  // whole warp past the end (uniform)
     bool active = e < n;
     if (key_off) {  // range mode: only [key_off[r] + hit[r], key_off[r+1])
         const int64_t total = R > 0 ? __ldg(key_off + R) : 0;
         bool in_range = false;
-        if ((int64_t)e0 < total) {
+        if (e0 < n && (int64_t)e0 < total) {
             const uint32_t r = pk::lane_request(key_off, R, (int64_t)e0, total, (int64_t)e);
             if ((int64_t)e < total) {
                 const int64_t h = __ldg(hit + r);
@@ -313,7 +316,9 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
         if (res < 0) set_status(status, res);
     }
     const uint32_t m = __ballot_sync(0xffffffffu, claimed_fast);
-    if (lane == 0 && m) atomicAdd(counter, (unsigned long long)__popc(m));
+    if (lane == 0 && m) atomicAdd_block(&block_claims, (unsigned long long)__popc(m));
+    __syncthreads();
+    if (threadIdx.x == 0 && block_claims) atomicAdd(counter, block_claims);
 }
 
 // Range mode for many short requests: one warp per request, no search.
@@ -325,16 +330,21 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
                   const uint32_t *__restrict__ slots, uint64_t n, const int64_t *__restrict__ key_off,
                   const int32_t *__restrict__ hit, uint32_t R, int32_t *__restrict__ result,
                   uint32_t *__restrict__ slot_out, int32_t *status) {
+    __shared__ unsigned long long block_claims;  // counted once per block (see k_store_claim)
+    if (threadIdx.x == 0) block_claims = 0;
+    __syncthreads();
     pk::pdl_launch_dependents();
     pk::pdl_wait();
     const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t lane = threadIdx.x & 31;
-    if (r >= R) return;  // uniform per warp
-    const int64_t a = __ldg(key_off + r);
-    int64_t b = __ldg(key_off + r + 1);
-    if ((uint64_t)b > n) b = (int64_t)n;
-    const int64_t h0 = __ldg(hit + r);
-    const int64_t first = a + (h0 > 0 ? h0 : 0);
+    int64_t a = 0, b = 0, first = 0;
+    if (r < R) {  // uniform per warp
+        a = __ldg(key_off + r);
+        b = __ldg(key_off + r + 1);
+        if ((uint64_t)b > n) b = (int64_t)n;
+        const int64_t h0 = __ldg(hit + r);
+        first = a + (h0 > 0 ? h0 : 0);
+    }
     unsigned long long cnt = 0;
     if (lane == 0) cnt = ld_volatile_u64(counter);
     const bool fast = __shfl_sync(0xffffffffu, cnt, 0) + n < capacity;
@@ -356,7 +366,9 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
         }
         claimed += __popc(__ballot_sync(0xffffffffu, claimed_fast));
     }
-    if (lane == 0 && claimed) atomicAdd(counter, (unsigned long long)claimed);
+    if (lane == 0 && claimed) atomicAdd_block(&block_claims, (unsigned long long)claimed);
+    __syncthreads();
+    if (threadIdx.x == 0 && block_claims) atomicAdd(counter, block_claims);
 }
 
 // Store, kernel 2 of 2: the lowest claimant of each new key writes its slot.
