@@ -160,7 +160,6 @@ __device__ __forceinline__ void load_tables(uint32_t *sK, uint32_t *sPad, const 
         sK[i] = pk::kSha256K[i];
         sPad[i] = pad.kw[i];
     }
-    if (threadIdx.x == 0) sK[64] = 1u;  // the multiplier of add_fma
 }
 
 // ---------------------------------------------------------------------------
@@ -189,7 +188,7 @@ __global__ void __launch_bounds__(kDigestBlock)
 k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_off,
                const int64_t *__restrict__ key_off, uint32_t R, uint32_t C, const __grid_constant__ PadKW pad,
                uint8_t *__restrict__ keys, const __grid_constant__ DescWork dw) {
-    __shared__ uint32_t sK[65], sPad[64];
+    __shared__ uint32_t sK[64], sPad[64];
     __shared__ __align__(16) uint32_t ring[kStages][kDigestBlock][16];
     pk::pdl_launch_dependents();
     if (blockIdx.x < dw.desc_blocks) {
@@ -252,7 +251,7 @@ k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ t
     const uint64_t bits = (uint64_t)C * 32u;
     const int rem = (int)(C % 16);
     if (rem == 0) {
-        pk::compress_kw(st, sPad, sK[64]);
+        pk::compress_kw(st, sPad);
     } else {
         const int32_t *tail = src + 16 * nfull;
 #pragma unroll
@@ -305,7 +304,6 @@ struct ChainSmem {
     uint32_t kw1[64][kChainLanes];     // block-1 K+W, t = 16..63 used
     uint32_t kw2[2][64][kChainLanes];  // block-2 K+W, double-buffered by step parity
     uint32_t kpub[8][kChainLanes];     // k_{i-1} for the schedule warp
-    uint32_t one;                      // the multiplier of pk::add_fma
 };
 
 // 16 schedule words t = 16q .. 16q+15 of the ring w (in place), K_t + W_t -> out[t][lane]
@@ -318,11 +316,10 @@ __device__ __forceinline__ void schedule16(uint32_t w[16], uint32_t (*out)[kChai
 }
 
 // rounds t = 16q .. 16q+15 with K+W from shared memory
-__device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint32_t (*kw)[kChainLanes], int q, uint32_t lane,
-                                            uint32_t one) {
+__device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint32_t (*kw)[kChainLanes], int q, uint32_t lane) {
     uint32_t a = v[0], b = v[1], c = v[2], d = v[3], e = v[4], f = v[5], g = v[6], h = v[7];
 #pragma unroll
-    for (int j = 0; j < 16; ++j) pk::round_kw(a, b, c, d, e, f, g, h, kw[16 * q + j][lane], one);
+    for (int j = 0; j < 16; ++j) pk::round_kw(a, b, c, d, e, f, g, h, kw[16 * q + j][lane]);
     v[0] = a; v[1] = b; v[2] = c; v[3] = d; v[4] = e; v[5] = f; v[6] = g; v[7] = h;
 }
 
@@ -330,12 +327,9 @@ __global__ void __launch_bounds__(2 * kChainLanes)
 k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_idx,
         const uint8_t *__restrict__ digests, uint32_t R, uint32_t D, uint8_t *keys) {
     __shared__ __align__(16) ChainSmem sm;
-    if (threadIdx.x == 0) sm.one = 1u;
-    __syncthreads();
     pk::pdl_launch_dependents();
     pk::pdl_wait();
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const uint32_t one = sm.one;
     const uint32_t r = blockIdx.x * kChainLanes + lane;
     int64_t a = 0, n = 0;
     uint32_t di = 0;
@@ -423,17 +417,17 @@ k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_i
         {   // block 1, rounds 0..15: W = k_{i-1} || d
             uint32_t a_ = v[0], b_ = v[1], c_ = v[2], d_ = v[3], e_ = v[4], f_ = v[5], g_ = v[6], h_ = v[7];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) pk::round_kw(a_, b_, c_, d_, e_, f_, g_, h_, pk::kSha256K[j] + p[j], one);
+            for (int j = 0; j < 8; ++j) pk::round_kw(a_, b_, c_, d_, e_, f_, g_, h_, pk::kSha256K[j] + p[j]);
 #pragma unroll
-            for (int j = 0; j < 8; ++j) pk::round_kw(a_, b_, c_, d_, e_, f_, g_, h_, kd[j], one);
+            for (int j = 0; j < 8; ++j) pk::round_kw(a_, b_, c_, d_, e_, f_, g_, h_, kd[j]);
             v[0] = a_; v[1] = b_; v[2] = c_; v[3] = d_; v[4] = e_; v[5] = f_; v[6] = g_; v[7] = h_;
         }
         bar_sync(1);
-        rounds16_kw(v, sm.kw1, 1, lane, one);
+        rounds16_kw(v, sm.kw1, 1, lane);
         bar_sync(2);
-        rounds16_kw(v, sm.kw1, 2, lane, one);
+        rounds16_kw(v, sm.kw1, 2, lane);
         bar_sync(3);
-        rounds16_kw(v, sm.kw1, 3, lane, one);
+        rounds16_kw(v, sm.kw1, 3, lane);
         uint32_t st[8] = {PK_IV0 + v[0], PK_IV1 + v[1], PK_IV2 + v[2], PK_IV3 + v[3],
                           PK_IV4 + v[4], PK_IV5 + v[5], PK_IV6 + v[6], PK_IV7 + v[7]};
         bar_sync(4);  // block-2 schedule of step i
@@ -441,7 +435,7 @@ k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_i
 #pragma unroll
         for (int j = 0; j < 8; ++j) v[j] = st[j];
 #pragma unroll 1
-        for (int q = 0; q < 4; ++q) rounds16_kw(v, kw2, q, lane, one);
+        for (int q = 0; q < 4; ++q) rounds16_kw(v, kw2, q, lane);
 #pragma unroll
         for (int j = 0; j < 8; ++j) p[j] = st[j] + v[j];
         if (i < n) store_digest(keys + 32ull * (a + i), p);

@@ -204,66 +204,44 @@ namespace pk {
 // loop of several compressions resident in the instruction cache; the round
 // constants are read from a shared-memory copy (sK, 64 words, see load_k).
 
-// x + y computed by the FMA pipe (IMAD x * 1 + y).  The logic and funnel
-// shift pipe is the bottleneck of SHA-256 on this SM; sums that are off the
-// round's critical path go to the otherwise idle multiply-add pipe.  The
-// factor is read from the (shared-memory) constant table so that the
-// compiler cannot fold the multiplication away.
-__device__ __forceinline__ uint32_t add_fma(uint32_t x, uint32_t y, uint32_t one) {
-    uint32_t r;
-    asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(r) : "r"(x), "r"(one), "r"(y));
-    return r;
-}
-
-// One round with K_t + W_t given.  h + kw and d + h + kw do not depend on the
-// previous round's e or a; the three sums that do stay 3-input adds.
 __device__ __forceinline__ void round_kw(uint32_t &a, uint32_t &b, uint32_t &c, uint32_t &d, uint32_t &e,
-                                         uint32_t &f, uint32_t &g, uint32_t &h, uint32_t kw, uint32_t one) {
-    const uint32_t hk = add_fma(h, kw, one);
-    const uint32_t dhk = add_fma(d, hk, one);
-    const uint32_t s1 = big_s1(e), c1 = ch(e, f, g);
-    const uint32_t en = dhk + s1 + c1;
-    const uint32_t t1 = hk + s1 + c1;
-    const uint32_t an = t1 + big_s0(a) + maj(a, b, c);
-    h = g; g = f; f = e; e = en; d = c; c = b; b = a; a = an;
+                                         uint32_t &f, uint32_t &g, uint32_t &h, uint32_t kw) {
+    const uint32_t t1 = h + big_s1(e) + ch(e, f, g) + kw;
+    const uint32_t t2 = big_s0(a) + maj(a, b, c);
+    h = g; g = f; f = e; e = d + t1; d = c; c = b; b = a; a = t1 + t2;
 }
 
 template <bool SCHED>
-__device__ __forceinline__ void rounds16(uint32_t v[8], uint32_t w[16], const uint32_t *__restrict__ k16,
-                                         uint32_t one) {
+__device__ __forceinline__ void rounds16(uint32_t v[8], uint32_t w[16], const uint32_t *__restrict__ k16) {
     uint32_t a = v[0], b = v[1], c = v[2], d = v[3], e = v[4], f = v[5], g = v[6], h = v[7];
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
-        if (SCHED)
-            w[j] = add_fma(w[j] + small_s1(w[(j + 14) & 15]), add_fma(w[(j + 9) & 15], small_s0(w[(j + 1) & 15]), one),
-                           one);
-        round_kw(a, b, c, d, e, f, g, h, add_fma(k16[j], w[j], one), one);
+        if (SCHED) w[j] += small_s1(w[(j + 14) & 15]) + w[(j + 9) & 15] + small_s0(w[(j + 1) & 15]);
+        round_kw(a, b, c, d, e, f, g, h, k16[j] + w[j]);
     }
     v[0] = a; v[1] = b; v[2] = c; v[3] = d; v[4] = e; v[5] = f; v[6] = g; v[7] = h;
 }
 
-// st <- st + compress(st, w); w is overwritten by the schedule.  sK holds the
-// 64 round constants followed by the word 1 (see add_fma).
+// st <- st + compress(st, w); w is overwritten by the schedule.
 __device__ __forceinline__ void compress_rolled(uint32_t st[8], uint32_t w[16], const uint32_t *__restrict__ sK) {
-    const uint32_t one = sK[64];
     uint32_t v[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) v[j] = st[j];
-    rounds16<false>(v, w, sK, one);
+    rounds16<false>(v, w, sK);
 #pragma unroll 1
-    for (int q = 1; q < 4; ++q) rounds16<true>(v, w, sK + 16 * q, one);
+    for (int q = 1; q < 4; ++q) rounds16<true>(v, w, sK + 16 * q);
 #pragma unroll
     for (int j = 0; j < 8; ++j) st[j] += v[j];
 }
 
 // st <- st + compress(st, W) for a message whose whole schedule is known in
-// advance: kw[t] = K_t + W_t for t = 0..63 (rounds only); one = 1.
-__device__ __forceinline__ void compress_kw(uint32_t st[8], const uint32_t *__restrict__ kw, uint32_t one) {
+// advance: kw[t] = K_t + W_t for t = 0..63 (rounds only).
+__device__ __forceinline__ void compress_kw(uint32_t st[8], const uint32_t *__restrict__ kw) {
     uint32_t a = st[0], b = st[1], c = st[2], d = st[3], e = st[4], f = st[5], g = st[6], h = st[7];
 #pragma unroll 1
     for (int q = 0; q < 4; ++q) {
 #pragma unroll
-        for (int j = 0; j < 16; ++j) round_kw(a, b, c, d, e, f, g, h, kw[16 * q + j], one);
+        for (int j = 0; j < 16; ++j) round_kw(a, b, c, d, e, f, g, h, kw[16 * q + j]);
     }
     st[0] += a; st[1] += b; st[2] += c; st[3] += d; st[4] += e; st[5] += f; st[6] += g; st[7] += h;
 }
