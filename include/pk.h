@@ -53,6 +53,7 @@ extern "C" {
 #define PK_ERR_PROBE_LIMIT (-6)    /* probe sequence longer than max_probe */
 #define PK_ERR_RESERVED_KEY (-7)   /* key prefix is all zero (the empty marker), p = 2^-128 */
 #define PK_ERR_CUDA (-8)           /* a CUDA runtime call or launch failed */
+#define PK_ERR_TOO_LARGE (-9)      /* n above PK_NOALLOC_MAX_ENTRIES (pk_store_noalloc only) */
 
 /* Per-entry store results (int32). Negative values are the error codes above. */
 #define PK_STORE_SKIPPED 0         /* not in a miss range (range mode) */
@@ -214,6 +215,37 @@ int pk_table_save(pk_ctx *ctx, void *dst, size_t dst_bytes, pk_stream stream);
  * pk_table_bytes + 64).  Keys and slots are restored exactly; the entries
  * count as inserted before any later store call.  Asynchronous on `stream`. */
 int pk_table_load(pk_ctx *ctx, const void *src, size_t src_bytes, pk_stream stream);
+
+/* Device.  The insert-if-absent of pk_store for callers that cannot allocate
+ * device memory and so cannot create a context (pk_init allocates the
+ * context's entry counter): code that runs while a CUDA graph is being
+ * captured, engines whose device memory is entirely owned by their own pool
+ * with a fixed budget, and latency-critical paths that must not enter the
+ * CUDA allocator.  The paper has no counterpart; this is an integration
+ * convenience.
+ * The table is described by cfg (table_dev, table_bytes, capacity_log2,
+ * max_probe; chunk_tokens is ignored) and must be all zero before its first
+ * use (cudaMemset, or a table created by pk_init).  Arguments, results and
+ * per-entry errors are those of pk_store, list or range mode.
+ * No memory is allocated: the call's scratch (the table's entry count, the
+ * latest call number in the table, and one 4-byte claim position per entry)
+ * is a fixed file-scope device array of 16 + 4 * PK_NOALLOC_MAX_ENTRIES bytes
+ * (about 1 MiB), held by every GPU that loads the library until the process
+ * exits.  n > PK_NOALLOC_MAX_ENTRIES returns PK_ERR_TOO_LARGE before
+ * anything is enqueued.  Each call first scans the whole table (count and
+ * latest call number), so its cost grows with the capacity.
+ * The first call on a device resolves the array's device address with
+ * cudaGetSymbolAddress (once per device, on the calling thread's current
+ * device); make that first call before any stream capture.
+ * All calls share the one array and it keeps the last call's contents: calls
+ * whose GPU work overlaps (other streams, other threads, the same device)
+ * race on it and must be serialised by the caller.  A table written by this
+ * entry point must not be written afterwards through pk_store of a context
+ * (their call numbers are not coordinated). */
+#define PK_NOALLOC_MAX_ENTRIES (1u << 18)
+int pk_store_noalloc(const pk_config *cfg, const uint8_t *keys_dev, const uint32_t *slots_dev, uint64_t n,
+                     const int64_t *key_off_dev, const int32_t *hit_chunks_dev, uint32_t R,
+                     int32_t *result_dev, uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream);
 
 /* Host, synchronous.  Number of entries in the table (device counter read
  * after synchronising `stream`). */

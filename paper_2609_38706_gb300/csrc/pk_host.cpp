@@ -269,6 +269,27 @@ int pk_table_load(pk_ctx *ctx, const void *src, size_t src_bytes, pk_stream stre
     return cuda_rc(pk_launch_mark_loaded(ctx, s));
 }
 
+int pk_store_noalloc(const pk_config *cfg, const uint8_t *keys_dev, const uint32_t *slots_dev, uint64_t n,
+                     const int64_t *key_off_dev, const int32_t *hit_chunks_dev, uint32_t R, int32_t *result_dev,
+                     uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream) {
+    if (!cfg || !cfg->table_dev || !aligned16(cfg->table_dev)) return PK_ERR_ARG;
+    const size_t need = pk_table_bytes(cfg->capacity_log2);
+    if (need == 0 || cfg->table_bytes < need) return PK_ERR_CAPACITY;
+    if ((key_off_dev == nullptr) != (hit_chunks_dev == nullptr)) return PK_ERR_ARG;
+    if (n > PK_NOALLOC_MAX_ENTRIES) return PK_ERR_TOO_LARGE;
+    if (n == 0) return PK_OK;
+    if (!keys_dev || !aligned16(keys_dev) || !slots_dev || !result_dev || !slot_out_dev) return PK_ERR_ARG;
+    if (!aligned(slots_dev, 4) || !aligned(result_dev, 4) || !aligned(slot_out_dev, 4) || !aligned(key_off_dev, 8) ||
+        !aligned(hit_chunks_dev, 4))
+        return PK_ERR_ARG;
+    const uint64_t capacity = 1ull << cfg->capacity_log2;
+    const uint32_t max_probe =
+        (cfg->max_probe == 0 || cfg->max_probe > capacity) ? (uint32_t)capacity : cfg->max_probe;
+    return cuda_rc(pk_launch_store_noalloc(static_cast<pk_entry *>(cfg->table_dev), cfg->capacity_log2, max_probe,
+                                           keys_dev, slots_dev, n, key_off_dev, hit_chunks_dev, R, result_dev,
+                                           slot_out_dev, status_dev, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 int pk_entries(pk_ctx *ctx, uint64_t *count, pk_stream stream) {
     if (!ctx || !count) return PK_ERR_ARG;
     unsigned long long v = 0;
@@ -291,6 +312,7 @@ const char *pk_strerror(int code) {
         case PK_ERR_PROBE_LIMIT: return "probe limit reached";
         case PK_ERR_RESERVED_KEY: return "key prefix is the reserved all-zero value";
         case PK_ERR_CUDA: return "CUDA runtime error";
+        case PK_ERR_TOO_LARGE: return "more entries than the allocation-free store's scratch holds (PK_NOALLOC_MAX_ENTRIES)";
         default: return "unknown status";
     }
 }

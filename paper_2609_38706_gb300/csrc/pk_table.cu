@@ -19,6 +19,8 @@
 #include "pk_device.cuh"
 #include "pk_internal.h"
 
+#include <mutex>
+
 namespace {
 
 using pk::set_status;
@@ -410,6 +412,114 @@ __global__ void k_mark_loaded(pk_entry *table, uint64_t capacity) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// Allocation-free store (pk_store_noalloc).  Same insert-if-absent as the
+// store above, for callers that own no libpk context: everything a context
+// would hold on the device (entry count, call number) and the per-entry claim
+// positions live in this one file-scope array, shared by every call.
+// ---------------------------------------------------------------------------
+struct NoallocScratch {
+    unsigned long long count;      // entries in the table (set by the scan, then claims)
+    unsigned long long epoch_max;  // largest call number found in the table
+    uint32_t pos[PK_NOALLOC_MAX_ENTRIES];  // table position of each PENDING entry
+};
+static __device__ __align__(256) NoallocScratch g_noalloc_scratch;
+
+// Count the occupied entries and find the latest call number in the table.
+__global__ void __launch_bounds__(256)
+k_noalloc_scan(const pk_entry *__restrict__ table, uint64_t capacity, NoallocScratch *sc) {
+    __shared__ unsigned long long blk_count, blk_epoch;
+    if (threadIdx.x == 0) blk_count = blk_epoch = 0;
+    __syncthreads();
+    unsigned long long cnt = 0, ep = 0;
+    for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < capacity;
+         i += (uint64_t)gridDim.x * blockDim.x) {
+        const uint4 k = __ldg(reinterpret_cast<const uint4 *>(table[i].k));
+        if (!is_zero(k)) {
+            ++cnt;
+            const unsigned long long e = __ldg(&table[i].epoch);
+            ep = e > ep ? e : ep;
+        }
+    }
+    atomicAdd_block(&blk_count, cnt);
+    atomicMax_block(&blk_epoch, ep);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        if (blk_count) atomicAdd(&sc->count, blk_count);
+        atomicMax(&sc->epoch_max, blk_epoch);
+    }
+}
+
+// One thread per entry (list or range mode), as k_store_claim; the call
+// number is one past the table's latest and PENDING positions go to scratch.
+__global__ void __launch_bounds__(256)
+k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity, NoallocScratch *sc,
+                const uint8_t *__restrict__ keys, const uint32_t *__restrict__ slots, uint64_t n,
+                const int64_t *__restrict__ key_off, const int32_t *__restrict__ hit, uint32_t R,
+                int32_t *__restrict__ result, uint32_t *__restrict__ slot_out, int32_t *status) {
+    __shared__ unsigned long long block_claims;
+    if (threadIdx.x == 0) block_claims = 0;
+    __syncthreads();
+    const unsigned long long epoch = ld_volatile_u64(&sc->epoch_max) + 1ull;
+    const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const uint32_t lane = threadIdx.x & 31;
+    const uint64_t e0 = e - lane;
+    bool active = e < n;
+    if (key_off) {
+        const int64_t total = R > 0 ? __ldg(key_off + R) : 0;
+        bool in_range = false;
+        if (e0 < n && (int64_t)e0 < total) {
+            const uint32_t r = pk::lane_request(key_off, R, (int64_t)e0, total, (int64_t)e);
+            if ((int64_t)e < total) {
+                const int64_t h = __ldg(hit + r);
+                in_range = (int64_t)e - __ldg(key_off + r) >= (h > 0 ? h : 0);
+            }
+        }
+        active = active && in_range;
+    }
+    unsigned long long cnt = 0;
+    if (lane == 0) cnt = ld_volatile_u64(&sc->count);
+    const bool fast = __shfl_sync(0xffffffffu, cnt, 0) + n < capacity;
+    int32_t res = PK_STORE_SKIPPED;
+    uint32_t out = PK_NO_SLOT;
+    bool claimed_fast = false;
+    if (active) {
+        const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
+        claim(table, mask, max_probe, capacity, &sc->count, epoch, fast, key, slots[e], e, res, out, claimed_fast);
+    }
+    if (e < n) {
+        result[e] = res;
+        if (res == PK_STORE_PENDING) {
+            sc->pos[e] = out;
+            slot_out[e] = PK_NO_SLOT;
+        } else {
+            slot_out[e] = out;
+        }
+        if (res < 0) set_status(status, res);
+    }
+    const uint32_t m = __ballot_sync(0xffffffffu, claimed_fast);
+    if (lane == 0 && m) atomicAdd_block(&block_claims, (unsigned long long)__popc(m));
+    __syncthreads();
+    if (threadIdx.x == 0 && block_claims) atomicAdd(&sc->count, block_claims);
+}
+
+__global__ void __launch_bounds__(256)
+k_noalloc_finalize(pk_entry *table, const NoallocScratch *sc, const uint32_t *__restrict__ slots, uint64_t n,
+                   int32_t *__restrict__ result, uint32_t *__restrict__ slot_out) {
+    const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= n || result[e] != PK_STORE_PENDING) return;
+    pk_entry *ent = table + sc->pos[e];
+    const uint32_t winner = ~ent->owner;
+    if (winner == (uint32_t)e) {
+        ent->slot = slots[e];
+        result[e] = PK_STORE_INSERTED;
+        slot_out[e] = slots[e];
+    } else {
+        result[e] = PK_STORE_PRESENT;
+        slot_out[e] = slots[winner];
+    }
+}
+
 unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1) / block); }
 
 // Per-request kernels when the batch has many short requests; per-key kernels
@@ -463,4 +573,41 @@ cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const u
     if (e == cudaSuccess)
         e = pk_launch(k_store_finalize, grid_for(n, 256), 256, s, ctx->table, slots, n, key_off, R, result, slot_out);
     return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// Device address of the allocation-free store's scratch array, resolved once
+// per device (host code cannot use the symbol's host-side name as an address).
+static void *noalloc_scratch_addr(int device) {
+    static std::mutex mu;
+    static void *addr[256] = {};
+    if (device < 0 || device >= 256) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[device]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+        addr[device] = p;
+    }
+    return addr[device];
+}
+
+cudaError_t pk_launch_store_noalloc(pk_entry *table, uint32_t capacity_log2, uint32_t max_probe,
+                                    const uint8_t *keys, const uint32_t *slots, uint64_t n, const int64_t *key_off,
+                                    const int32_t *hit_chunks, uint32_t R, int32_t *result, uint32_t *slot_out,
+                                    int32_t *status, cudaStream_t s) {
+    int device = -1;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e != cudaSuccess) return e;
+    NoallocScratch *sc = static_cast<NoallocScratch *>(noalloc_scratch_addr(device));
+    if (!sc) return cudaErrorInvalidSymbol;
+    if (n == 0) return cudaSuccess;
+    const uint64_t capacity = 1ull << capacity_log2;
+    // count and epoch_max must start at zero; pos needs no clearing
+    e = cudaMemsetAsync(sc, 0, 2 * sizeof(unsigned long long), s);
+    if (e != cudaSuccess) return e;
+    const uint64_t scan_blocks = (capacity + 255) / 256;
+    k_noalloc_scan<<<(unsigned)(scan_blocks < 152 * 8 ? scan_blocks : 152 * 8), 256, 0, s>>>(table, capacity, sc);
+    k_noalloc_claim<<<grid_for(n, 256), 256, 0, s>>>(table, capacity - 1, max_probe, capacity, sc, keys, slots, n,
+                                                      key_off, hit_chunks, key_off ? R : 0, result, slot_out, status);
+    k_noalloc_finalize<<<grid_for(n, 256), 256, 0, s>>>(table, sc, slots, n, result, slot_out);
+    return cudaGetLastError();
 }

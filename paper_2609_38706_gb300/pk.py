@@ -26,6 +26,8 @@ PK_ERR_TABLE_FULL = -5
 PK_ERR_PROBE_LIMIT = -6
 PK_ERR_RESERVED_KEY = -7
 PK_ERR_CUDA = -8
+PK_ERR_TOO_LARGE = -9
+PK_NOALLOC_MAX_ENTRIES = 1 << 18
 PK_STORE_SKIPPED = 0
 PK_STORE_INSERTED = 1
 PK_STORE_PRESENT = 2
@@ -85,6 +87,8 @@ def lib() -> ctypes.CDLL:
             "pk_lookup": (ctypes.c_int, [_VP, _VP, _VP, _U32, _U64, _VP, _VP, _VP, _VP]),
             "pk_store": (ctypes.c_int, [_VP, _VP, _VP, _U64, _VP, _VP, _U32, _VP, _VP, _VP, _VP]),
             "pk_entries": (ctypes.c_int, [_VP, ctypes.POINTER(ctypes.c_uint64), _VP]),
+            "pk_store_noalloc": (ctypes.c_int, [ctypes.POINTER(pk_config), _VP, _VP, _U64, _VP, _VP, _U32, _VP, _VP,
+                                                _VP, _VP]),
             "pk_table_save": (ctypes.c_int, [_VP, _VP, ctypes.c_size_t, _VP]),
             "pk_table_load": (ctypes.c_int, [_VP, _VP, ctypes.c_size_t, _VP]),
             "pk_strerror": (ctypes.c_char_p, [ctypes.c_int]),
@@ -265,6 +269,19 @@ def pk_table_save(ctx: int, dst: torch.Tensor, stream=None) -> None:
 
 def pk_table_load(ctx: int, src: torch.Tensor, stream=None) -> None:
     _check(lib().pk_table_load(ctx, _p(src), src.numel() * src.element_size(), _s(stream)), "pk_table_load")
+
+
+def pk_store_noalloc(table: torch.Tensor, capacity_log2: int, keys: torch.Tensor, slots: torch.Tensor,
+                     result: torch.Tensor, slot_out: torch.Tensor, status: torch.Tensor, max_probe: int = 0,
+                     key_off: Optional[torch.Tensor] = None, hit_chunks: Optional[torch.Tensor] = None,
+                     stream=None) -> None:
+    """pk_store without a context, for callers that cannot allocate device
+    memory; the table tensor must be zero-filled before its first use."""
+    cfg = pk_config(1, capacity_log2, max_probe, _p(table), table.numel() * table.element_size())
+    n = keys.numel() // 32
+    R = 0 if key_off is None else key_off.numel() - 1
+    _check(lib().pk_store_noalloc(ctypes.byref(cfg), _p(keys), _p(slots), n, _p(key_off), _p(hit_chunks), R,
+                                  _p(result), _p(slot_out), _p(status), _s(stream)), "pk_store_noalloc")
 
 
 def pk_entries(ctx: int, stream=None) -> int:
