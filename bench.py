@@ -51,6 +51,33 @@ def load_peaks():
     return {"hbm_gbs": 6800.0, "sm_max_mhz": 2070.0, "source": "fallback"}
 
 
+DERIVE_SOURCES = ("paper_2609_38706_gb300/csrc/pk_derive.cu", "paper_2609_38706_gb300/csrc/pk_sha256.cuh",
+                  "paper_2609_38706_gb300/csrc/pk_device.cuh", "paper_2609_38706_gb300/csrc/pk_internal.h")
+
+
+def derive_traffic(workload: str):
+    """Cold-cache DRAM bytes of one key-derivation call, from the committed ncu
+    summary, or None when the kernels changed since it was taken (or another
+    workload is run)."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in DERIVE_SOURCES:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    fields = {}
+    try:
+        with open(os.path.join(ROOT, "profiles", "dram_traffic_multi_adapter.md")) as fh:
+            for line in fh:
+                k, _, v = line.strip().partition(":")
+                if v:
+                    fields[k.strip()] = v.strip()
+    except OSError:
+        return None
+    if fields.get("kernel_sources_sha256") != h.hexdigest() or fields.get("workload") != workload:
+        return None
+    return int(fields["derive_traffic_bytes_per_call"])
+
+
 def compressions(n_keys: int, C: int) -> tuple[int, int]:
     """SHA-256 compressions per batch: chunk digests (ceil((4C + 9) / 64) each)
     and chain steps (a 96-byte message = 2 each)."""
@@ -360,7 +387,11 @@ def main():
     peaks = load_peaks()
     c_dig, c_chain = compressions(n_keys, C)
     derive_s = float(np.mean(derive_ms)) / 1e3
-    alu_peak = SMS * LANES_PER_SM * peaks["sm_max_mhz"] * 1e6 / 1e12           # Tops/s
+    alu_peak = SMS * LANES_PER_SM * peaks["sm_max_mhz"] * 1e6 / 1e12           # Tops/s, issue-rate ceiling
+    # the logic/shift pipe takes 16 lanes per sub-partition per clock and SHA-256 with funnel-shift
+    # rotations needs 1024 of its operations per compression (6 SHF + 4 LOP3 per round, 6 + 2 per
+    # schedule word): the ceiling for this formulation, in the same 1384-op units
+    alu_pipe_peak = SMS * 64 * peaks["sm_max_mhz"] * 1e6 / 1024 * SHA_OPS_PER_COMPRESSION / 1e12
     achieved = (c_dig + c_chain) * SHA_OPS_PER_COMPRESSION / derive_s / 1e12
     lookup_s = float(np.mean(lookup_ms)) / 1e3
     probe_bytes = n_keys * (16 + 32 + 4) + R * 4
@@ -376,7 +407,9 @@ def main():
         "roofline": {"bound": "alu",
                      "kernel": "pk_derive_keys_enc (chunk offsets; chunk + descriptor digests; chain)",
                      "achieved": achieved, "peak": alu_peak, "unit": "Tops/s", "frac": achieved / alu_peak,
-                     "traffic": None,
+                     "traffic": derive_traffic(args.workload),
+                     "algorithmic_bytes": wl.batch.n_tokens * 4 + n_keys * 32,
+                     "alu_pipe_peak": alu_pipe_peak,
                      "peak_basis": f"{SMS} SMs x {LANES_PER_SM} int32 lanes x {peaks['sm_max_mhz']:.0f} MHz "
                                    f"(issue-rate ceiling); {SHA_OPS_PER_COMPRESSION} ops per compression, "
                                    f"{c_dig + c_chain} compressions per launch"},
