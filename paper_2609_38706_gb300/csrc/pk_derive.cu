@@ -62,67 +62,79 @@ k_digest_descriptors(const uint8_t *__restrict__ enc, uint64_t enc_bytes, const 
 }
 
 // ---------------------------------------------------------------------------
-// Chunk offsets: one block.  Validates the request layout, then writes the
-// exclusive scan of floor(T_r / C).  Any invalid request zeroes all offsets.
+// Chunk offsets: one block, requests in tiles of kScanThreads * kScanItems.
+// Each thread takes kScanItems consecutive requests of the tile (coalesced
+// offset loads), the block scans the per-thread sums, and a running carry
+// links the tiles.  Any invalid request (offsets decreasing, negative or past
+// n_tokens, descriptor index >= D) or a total above key_capacity zeroes all
+// offsets afterwards and reports PK_ERR_ARG.
 // ---------------------------------------------------------------------------
 constexpr int kScanThreads = 1024;
+constexpr int kScanItems = 4;
 
 __global__ void __launch_bounds__(kScanThreads)
 k_chunk_offsets(const int64_t *__restrict__ tok_off, uint32_t R, uint64_t n_tokens, uint32_t C,
                 const uint32_t *__restrict__ desc_idx, uint32_t D, uint64_t key_capacity,
                 int64_t *__restrict__ key_off, int32_t *status) {
     __shared__ long long warp_sums[kScanThreads / 32];
-    __shared__ long long total_s;
+    __shared__ long long tile_total;
     pk::pdl_launch_dependents();
     pk::pdl_wait();
-    const uint32_t tid = threadIdx.x;
-    const uint64_t per = (R + kScanThreads - 1) / kScanThreads;
-    const uint64_t lo = tid * per;
-    const uint64_t hi = lo + per < R ? lo + per : R;
-
+    const uint32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (tid == 0) key_off[0] = 0;
     bool bad = false;
-    long long local = 0;
-    for (uint64_t r = lo; r < hi; ++r) {
-        const int64_t a = tok_off[r], b = tok_off[r + 1];
-        if (a < 0 || b < a || (uint64_t)b > n_tokens || desc_idx[r] >= D) bad = true;
-        else local += (b - a) / C;
-    }
-    bad = __syncthreads_or(bad);
-
-    // block exclusive scan of the per-thread sums
-    const int lane = tid & 31, warp = tid >> 5;
-    long long incl = local;
+    long long carry = 0;
+    for (uint64_t base = 0; base < R; base += (uint64_t)kScanThreads * kScanItems) {
+        const uint64_t r0 = base + (uint64_t)tid * kScanItems;
+        long long n[kScanItems];
+        long long local = 0;
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const long long v = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += v;
-    }
-    if (lane == 31) warp_sums[warp] = incl;
-    __syncthreads();
-    if (warp == 0) {
-        long long ws = warp_sums[lane];
-        long long wincl = ws;
+        for (int j = 0; j < kScanItems; ++j) {
+            const uint64_t r = r0 + j;
+            n[j] = 0;
+            if (r < R) {
+                const int64_t a = tok_off[r], b = tok_off[r + 1];
+                if (a < 0 || b < a || (uint64_t)b > n_tokens || desc_idx[r] >= D) bad = true;
+                else n[j] = (b - a) / C;
+            }
+            local += n[j];
+        }
+        // block exclusive scan of the per-thread sums
+        long long incl = local;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-            const long long v = __shfl_up_sync(0xffffffffu, wincl, o);
-            if (lane >= o) wincl += v;
+            const long long v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
         }
-        warp_sums[lane] = wincl - ws;
-        if (lane == 31) total_s = wincl;
+        if (lane == 31) warp_sums[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            const long long ws = warp_sums[lane];
+            long long wincl = ws;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const long long v = __shfl_up_sync(0xffffffffu, wincl, o);
+                if (lane >= o) wincl += v;
+            }
+            warp_sums[lane] = wincl - ws;
+            if (lane == 31) tile_total = wincl;
+        }
+        __syncthreads();
+        long long run = carry + warp_sums[warp] + incl - local;
+#pragma unroll
+        for (int j = 0; j < kScanItems; ++j) {
+            if (r0 + j < R) {
+                run += n[j];
+                key_off[r0 + j + 1] = run;
+            }
+        }
+        carry += tile_total;
+        __syncthreads();  // warp_sums and tile_total are reused by the next tile
     }
-    __syncthreads();
-    long long run = warp_sums[warp] + incl - local;
-    const bool too_many = (unsigned long long)total_s > key_capacity;
-
-    if (tid == 0) key_off[0] = 0;
-    if (bad || too_many) {
-        for (uint64_t r = lo; r < hi; ++r) key_off[r + 1] = 0;
+    bad = __syncthreads_or(bad);
+    if (bad || (unsigned long long)carry > key_capacity) {
+        for (uint64_t r = tid; r < R; r += kScanThreads) key_off[r + 1] = 0;
         if (tid == 0) set_status(status, PK_ERR_ARG);
-        return;
-    }
-    for (uint64_t r = lo; r < hi; ++r) {
-        run += (tok_off[r + 1] - tok_off[r]) / C;
-        key_off[r + 1] = run;
     }
 }
 
@@ -172,43 +184,11 @@ __device__ __forceinline__ void load_tables(uint32_t *sK, uint32_t *sPad, const 
 constexpr int kDigestBlock = 128;
 constexpr int kStages = 3;
 
-// Optional descriptor work for the same launch (fused a0): the first
-// desc_blocks blocks hash descriptor encodings instead, one warp each.
-struct DescWork {
-    const uint8_t *enc;
-    uint64_t enc_bytes;
-    const int64_t *enc_off;
-    uint32_t D;
-    uint8_t *digests;
-    int32_t *status;
-    uint32_t desc_blocks;
-};
-
-__global__ void __launch_bounds__(kDigestBlock)
-k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_off,
-               const int64_t *__restrict__ key_off, uint32_t R, uint32_t C, const __grid_constant__ PadKW pad,
-               uint8_t *__restrict__ keys, const __grid_constant__ DescWork dw) {
-    __shared__ uint32_t sK[64], sPad[64];
-    __shared__ __align__(16) uint32_t ring[kStages][kDigestBlock][16];
-    pk::pdl_launch_dependents();
-    if (blockIdx.x < dw.desc_blocks) {
-        pk::pdl_wait();
-        const uint32_t warp = threadIdx.x >> 5;
-        const uint32_t j = blockIdx.x * (kDigestBlock / 32) + warp;
-        uint8_t *stage = reinterpret_cast<uint8_t *>(ring[0]) + warp * kDescStage;  // 4 x 2 KiB of the ring
-        if (j < dw.D) hash_descriptor(stage, dw.enc, dw.enc_bytes, dw.enc_off, j, dw.digests, dw.status);
-        return;
-    }
-    load_tables(sK, sPad, pad);
-    __syncthreads();
-    pk::pdl_wait();
-    if (R == 0) return;
-    const int64_t g = (int64_t)(blockIdx.x - dw.desc_blocks) * blockDim.x + threadIdx.x;
-    const int64_t g0 = g - (threadIdx.x & 31);
-    const int64_t total = __ldg(key_off + R);
-    if (g0 >= total) return;  // whole warp past the end
-    const uint32_t r = pk::lane_request(key_off, R, g0, total, g);
-    if (g >= total) return;
+// c = SHA-256 of chunk g (request r), written to keys[g].
+__device__ __forceinline__ void digest_chunk(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_off,
+                                             const int64_t *__restrict__ key_off, uint32_t r, int64_t g, uint32_t C,
+                                             const uint32_t *sK, const uint32_t *sPad,
+                                             uint32_t (*ring)[kDigestBlock][16], uint8_t *__restrict__ keys) {
     const int64_t i = g - __ldg(key_off + r);
     const int32_t *src = tokens + __ldg(tok_off + r) + i * (int64_t)C;
     const bool aligned = (reinterpret_cast<uintptr_t>(src) & 15) == 0;
@@ -273,6 +253,51 @@ k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ t
     store_digest(keys + 32 * g, st);
 }
 
+// Optional descriptor work for the same launch (fused a0): the first
+// desc_blocks blocks hash descriptor encodings instead, one warp each.
+struct DescWork {
+    const uint8_t *enc;
+    uint64_t enc_bytes;
+    const int64_t *enc_off;
+    uint32_t D;
+    uint8_t *digests;
+    int32_t *status;
+    uint32_t desc_blocks;
+};
+
+__global__ void __launch_bounds__(kDigestBlock)
+k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_off,
+               const int64_t *__restrict__ key_off, uint32_t R, uint32_t C, const __grid_constant__ PadKW pad,
+               uint8_t *__restrict__ keys, const __grid_constant__ DescWork dw, uint32_t r_begin, uint32_t r_end) {
+    __shared__ uint32_t sK[64], sPad[64];
+    __shared__ __align__(16) uint32_t ring[kStages][kDigestBlock][16];
+    pk::pdl_launch_dependents();
+    if (blockIdx.x < dw.desc_blocks) {
+        pk::pdl_wait();
+        const uint32_t warp = threadIdx.x >> 5;
+        const uint32_t j = blockIdx.x * (kDigestBlock / 32) + warp;
+        uint8_t *stage = reinterpret_cast<uint8_t *>(ring[0]) + warp * kDescStage;  // 4 x 2 KiB of the ring
+        if (j < dw.D) hash_descriptor(stage, dw.enc, dw.enc_bytes, dw.enc_off, j, dw.digests, dw.status);
+        return;
+    }
+    load_tables(sK, sPad, pad);
+    __syncthreads();
+    pk::pdl_wait();
+    if (R == 0 || r_begin >= r_end) return;
+    // the chunks of requests [r_begin, r_end), in tiles of one block, grid-strided
+    const int64_t g_begin = __ldg(key_off + r_begin), g_end = __ldg(key_off + r_end);
+    const uint32_t nblocks = gridDim.x - dw.desc_blocks;
+    for (int64_t tile = g_begin + (int64_t)(blockIdx.x - dw.desc_blocks) * kDigestBlock; tile < g_end;
+         tile += (int64_t)nblocks * kDigestBlock) {
+        const int64_t g = tile + threadIdx.x;
+        const int64_t g0 = g - (threadIdx.x & 31);
+        if (g0 >= g_end) break;  // whole warp past the end (uniform per warp)
+        const uint32_t r = pk::lane_request(key_off, R, g0, g_end, g);
+        if (g < g_end) digest_chunk(tokens, tok_off, key_off, r, g, C, sK, sPad, ring, keys);
+        __syncwarp();
+    }
+}
+
 // ---------------------------------------------------------------------------
 // Chain: k_i = SHA-256(k_{i-1} || d || c_i), serial in i for each request.
 //
@@ -325,12 +350,12 @@ __device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint32_t (*kw)[
 
 __global__ void __launch_bounds__(2 * kChainLanes)
 k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_idx,
-        const uint8_t *__restrict__ digests, uint32_t R, uint32_t D, uint8_t *keys) {
+        const uint8_t *__restrict__ digests, uint32_t r_begin, uint32_t R, uint32_t D, uint8_t *keys) {
     __shared__ __align__(16) ChainSmem sm;
     pk::pdl_launch_dependents();
     pk::pdl_wait();
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const uint32_t r = blockIdx.x * kChainLanes + lane;
+    const uint32_t r = r_begin + blockIdx.x * kChainLanes + lane;  // requests [r_begin, R)
     int64_t a = 0, n = 0;
     uint32_t di = 0;
     if (r < R) {
@@ -482,19 +507,20 @@ cudaError_t pk_launch_derive_enc(const pk_ctx *ctx, const int32_t *tokens, uint6
     if (e != cudaSuccess) return e;
     DescWork dw = {enc, enc_bytes, enc_off, D, digests, status, 0};
     if (enc_off) dw.desc_blocks = grid_for(D, kDigestBlock / 32);
+    PadKW pad;
+    for (int t = 0; t < 64; ++t) pad.kw[t] = ctx->pad_kw[t];
     const bool chunks = R > 0 && key_capacity > 0;
-    const unsigned digest_blocks = chunks ? grid_for(key_capacity, kDigestBlock) : 0;
-    if (digest_blocks + dw.desc_blocks > 0) {
-        PadKW pad;
-        for (int t = 0; t < 64; ++t) pad.kw[t] = ctx->pad_kw[t];
-        e = pk_launch(k_chunk_digest, digest_blocks + dw.desc_blocks, kDigestBlock, s, tokens, tok_off,
-                      (const int64_t *)key_off, R, C, pad, keys, dw);
-        if (e != cudaSuccess) return e;
+    if (!chunks) {
+        if (dw.desc_blocks)
+            e = pk_launch(k_chunk_digest, dw.desc_blocks, kDigestBlock, s, tokens, tok_off, (const int64_t *)key_off, R,
+                          C, pad, keys, dw, 0u, 0u);
+        return e != cudaSuccess ? e : cudaGetLastError();
     }
-    if (chunks) {
-        e = pk_launch(k_chain, grid_for(R, kChainLanes), 2 * kChainLanes, s, (const int64_t *)key_off, desc_idx,
-                      (const uint8_t *)digests, R, D, keys);
-        if (e != cudaSuccess) return e;
-    }
+    e = pk_launch(k_chunk_digest, grid_for(key_capacity, kDigestBlock) + dw.desc_blocks, kDigestBlock, s, tokens,
+                  tok_off, (const int64_t *)key_off, R, C, pad, keys, dw, 0u, R);
+    if (e != cudaSuccess) return e;
+    e = pk_launch(k_chain, grid_for(R, kChainLanes), 2 * kChainLanes, s, (const int64_t *)key_off, desc_idx,
+                  (const uint8_t *)digests, 0u, R, D, keys);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

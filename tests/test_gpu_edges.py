@@ -215,3 +215,18 @@ def test_descriptor_digest_device_equals_host_and_oracle():
     assert np.array_equal(dg, O.descriptor_digests(descs))
     assert all(pk.pk_descriptor_digest(d) == dg[j].tobytes() for j, d in enumerate(descs))
     kt.close()
+
+
+@pytest.mark.parametrize("R,C", [(9000, 16), (5000, 7)])
+def test_many_requests_span_scan_tiles_and_parts(R, C):
+    """More requests than one scan tile (4096) and enough chunks for the
+    overlapped multi-part derivation; ragged lengths and empty requests."""
+    rng = np.random.default_rng(R + C)
+    lens = rng.integers(0, 40 * C, R)
+    lens[::13] = 0
+    rows = [rng.integers(0, 152064, int(n)).astype(np.int32) for n in lens]
+    descs = [DESC, dict(DESC, salt="a"), dict(DESC, adapter_id="adapter-07")]
+    kt = KT(C, log2=10)
+    ko, keys, rko, rkeys = derive_both(kt, rows, rng.integers(0, 3, R), descs, C)
+    assert np.array_equal(ko, rko) and np.array_equal(keys, rkeys)
+    kt.close()
