@@ -47,54 +47,182 @@ __device__ __forceinline__ unsigned long long ld_volatile_u64(const unsigned lon
     return v;
 }
 
-// Entries are examined in windows of up to kWin consecutive entries (one
-// 128-byte line, aligned): the keys of a window are loaded together, so a
-// probe sequence costs one memory round trip per window instead of one per
-// entry.  The examination order is still home, home+1, ... as in plain
-// linear probing.
+// Cooperative probing.  A warp probes the keys of its lanes together.  In
+// each round the m keys still undecided are spread over the 32 lanes,
+// G = 2^floor(log2(32/m)) lanes per key, and lane j of a key's group loads
+// the j-th window of the key's remaining probe sequence: kWin consecutive
+// entries (one aligned 128-byte line).  One ballot then finds, in sequence
+// order, the first entry that decides the key (its own key, or an empty
+// entry).  With a full warp of keys every lane reads one window per round,
+// as a lane-per-key probe would; a key whose sequence runs long is joined by
+// the lanes whose keys are done, so the warp no longer waits one round trip
+// per window for its slowest key.  The entries examined and the decision
+// are those of plain linear probing, home, home+1, ...; only the number of
+// windows loaded at once differs.
 constexpr uint32_t kWin = 4;
+constexpr uint32_t kFull = 0xffffffffu;
+
+__device__ __forceinline__ uint32_t lanemask_lt() {
+    uint32_t m;
+    asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+    return m;
+}
+
+// Position of the set bit of rank n (0-based, from bit 0) of mask; n < popc(mask).
+__device__ __forceinline__ uint32_t nth_set_bit(uint32_t mask, uint32_t n) {
+    uint32_t pos = 0;
+#pragma unroll
+    for (uint32_t s = 16; s >= 1; s >>= 1) {
+        const uint32_t low = __popc(mask & ((1u << s) - 1u));
+        if (n >= low) {
+            n -= low;
+            mask >>= s;
+            pos += s;
+        }
+    }
+    return pos;
+}
+
+__device__ __forceinline__ uint4 shfl4(const uint4 &v, uint32_t src) {
+    return make_uint4(__shfl_sync(kFull, v.x, src), __shfl_sync(kFull, v.y, src), __shfl_sync(kFull, v.z, src),
+                      __shfl_sync(kFull, v.w, src));
+}
+
+// Read-only 16-byte load kept in program order (prefetch of the next keys).
+__device__ __forceinline__ uint4 ld_nc_v4(const void *p) {
+    uint4 v;
+    asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
+// This lane's roles in one round, given the mask P of lanes whose key is
+// still undecided.
+struct Round {
+    uint32_t G;          // lanes per undecided key (power of two)
+    uint32_t j;          // worker role: window index within its group
+    uint32_t owner;      // worker role: lane holding the key it works on
+    bool work;           // worker role: has a key to work on
+    uint32_t work_mask;  // lanes of the group it works in
+    uint32_t own_mask;   // owner role: lanes working on its own key
+};
+
+__device__ __forceinline__ Round plan_round(uint32_t P, uint32_t lane) {
+    Round r;
+    const uint32_t m = __popc(P);  // >= 1
+    const uint32_t lg = 31 - __clz(32u / m);
+    r.G = 1u << lg;
+    const uint32_t gm = lg == 5 ? kFull : (1u << r.G) - 1u;
+    const uint32_t q = lane >> lg;
+    r.j = lane & (r.G - 1);
+    r.work = q < m;
+    r.owner = r.work ? nth_set_bit(P, q) : lane;
+    r.work_mask = gm << (q << lg);
+    const uint32_t qo = __popc(P & lanemask_lt());
+    r.own_mask = ((P >> lane) & 1u) ? gm << (qo << lg) : 0u;
+    return r;
+}
+
+// Window geometry of a probe position: the aligned window holding it and
+// the offset of the position in it.
+__device__ __forceinline__ uint32_t window_size(uint64_t mask) { return mask + 1 < kWin ? (uint32_t)(mask + 1) : kWin; }
+
+// A lane's key while it is being probed (owner role).
+struct ProbeKey {
+    uint4 key;
+    uint64_t e;       // entry index of the key in the caller's arrays
+    uint64_t pos;     // next table position of its probe sequence
+    uint32_t probed;  // entries of the sequence examined so far
+    bool pending;     // not decided yet
+};
+
+__device__ __forceinline__ void probe_start(ProbeKey &s, const uint4 &key, uint64_t e, uint64_t mask) {
+    s.key = key;
+    s.e = e;
+    s.pos = home_of(key) & mask;
+    s.probed = 0;
+    s.pending = true;
+}
+
+// Owner role after a round in which no lane of its group found a deciding
+// entry: the key's sequence continues after the group's G windows.
+__device__ __forceinline__ void skip_windows(ProbeKey &s, uint32_t G, uint32_t win, uint64_t mask) {
+    const uint64_t b0 = s.pos & ~(uint64_t)(win - 1);
+    s.probed += G * win - (uint32_t)(s.pos - b0);
+    s.pos = (b0 + (uint64_t)G * win) & mask;
+}
 
 // ---------------------------------------------------------------------------
-// Lookup of one key: its slot, or PK_NO_SLOT.  Returns false if the probe
-// sequence reached max_probe without an answer.
+// Lookup: one round over the undecided keys P of the warp.  Returns true in
+// the lanes whose key was decided in this round, with its slot (PK_NO_SLOT
+// if absent) and `limit` set if its sequence reached max_probe.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ bool probe(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
-                                      const uint4 &key, uint32_t &slot) {
-    slot = PK_NO_SLOT;
-    if (is_zero(key)) return true;  // the empty marker is never stored
-    const uint32_t win = mask + 1 < kWin ? (uint32_t)(mask + 1) : kWin;
-    const uint64_t pos = home_of(key) & mask;
-    uint64_t base = pos & ~(uint64_t)(win - 1);
-    uint32_t j0 = (uint32_t)(pos - base);
-    uint32_t probed = 0;
-    bool done = false;
-    while (!done && probed < max_probe) {
-        const pk_entry *grp = table + base;
+__device__ __forceinline__ bool lookup_round(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
+                                             uint32_t P, ProbeKey &s, uint32_t &slot, bool &limit) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t win = window_size(mask);
+    // With every lane's key undecided (the common case while a request has
+    // keys left) each lane probes its own key and nothing is exchanged.
+    const bool full = P == kFull;
+    const Round rd = full ? Round{1, 0, lane, true, 1u << lane, 1u << lane} : plan_round(P, lane);
+    const uint4 k = full ? s.key : shfl4(s.key, rd.owner);
+    const uint64_t wpos = full ? s.pos : __shfl_sync(kFull, s.pos, rd.owner);
+    const uint32_t wprobed = full ? s.probed : __shfl_sync(kFull, s.probed, rd.owner);
+    const uint64_t base0 = wpos & ~(uint64_t)(win - 1);
+    const uint32_t j0 = (uint32_t)(wpos - base0);
+    const uint64_t wb = (base0 + (uint64_t)rd.j * win) & mask;
+    int cand = -1;
+    bool match = false;
+    if (rd.work) {
+        const pk_entry *grp = table + wb;
         uint4 v[kWin];
 #pragma unroll
-        for (uint32_t u = 0; u < kWin; ++u)
-            if (u < win) v[u] = __ldg(reinterpret_cast<const uint4 *>(grp[u].k));
+        for (uint32_t u = 0; u < kWin; ++u) {  // entries before the sequence start are not read
+            v[u] = make_uint4(0, 0, 0, 0);
+            if (u < win && (rd.j > 0 || u >= j0)) v[u] = __ldg(reinterpret_cast<const uint4 *>(grp[u].k));
+        }
 #pragma unroll
         for (uint32_t u = 0; u < kWin; ++u) {
-            if (u < win && u >= j0 && !done && probed < max_probe) {
-                ++probed;
-                if (same(v[u], key)) {
-                    slot = __ldg(&grp[u].slot);
-                    done = true;
+            const bool in_seq = u < win && (rd.j > 0 || u >= j0) && wprobed + (rd.j * win + u - j0) < max_probe;
+            if (in_seq && cand < 0) {
+                if (same(v[u], k)) {
+                    cand = (int)u;
+                    match = true;
                 } else if (is_zero(v[u])) {
-                    done = true;
+                    cand = (int)u;
                 }
             }
         }
-        base = (base + win) & mask;
-        j0 = 0;
     }
-    return done;
+    const uint32_t B = __ballot_sync(kFull, cand >= 0);
+    const bool decider = cand >= 0 && (B & rd.work_mask & lanemask_lt()) == 0;
+    uint32_t dslot = PK_NO_SLOT;
+    if (decider && match) dslot = __ldg(&table[wb + (uint32_t)cand].slot);
+    const uint32_t ob = B & rd.own_mask;
+    const uint32_t got = full ? dslot : __shfl_sync(kFull, dslot, ob ? __ffs(ob) - 1 : lane);
+    if (!s.pending) return false;
+    if (ob) {
+        slot = got;
+        limit = false;
+        s.pending = false;
+        return true;
+    }
+    skip_windows(s, rd.G, win, mask);
+    if (s.probed >= max_probe) {
+        slot = PK_NO_SLOT;
+        limit = true;
+        s.pending = false;
+        return true;
+    }
+    return false;
 }
 
-// One warp per request: every key's slot, and h_r = index of the first miss
-// (ballot over each group of 32 keys).  For batches of many short requests.
-__global__ void __launch_bounds__(256)
+// One warp per request: every key's slot, and h_r = index of the first miss.
+// A lane whose key is decided takes the request's next key, from a register
+// buffer holding the next 32 keys (loaded one refill ahead), so the warp
+// keeps 32 keys in flight until the request's last keys.
+__global__ void __launch_bounds__(256, 4)
 k_lookup_req(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
              const uint8_t *__restrict__ keys, const int64_t *__restrict__ key_off, uint32_t R,
              uint64_t key_capacity, uint32_t *__restrict__ slots, int32_t *__restrict__ hit, int32_t *status) {
@@ -106,25 +234,55 @@ k_lookup_req(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_pro
     const int64_t a = __ldg(key_off + r);
     int64_t b = __ldg(key_off + r + 1);
     if ((uint64_t)b > key_capacity) b = (int64_t)key_capacity;
-    int64_t h = -1;
+    uint32_t first_miss = 0xffffffffu;  // lowest missing index (relative to a) seen by this lane
     bool limit = false;
-    for (int64_t base = a; base < b; base += 32) {
-        const int64_t g = base + lane;
-        uint32_t slot = PK_NO_SLOT;
-        if (g < b) {
-            const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * g));
-            if (!probe(table, mask, max_probe, key, slot)) limit = true;
-            slots[g] = slot;
+    ProbeKey s;
+    s.pending = false;
+    bool busy = false;  // holds a key (pending)
+    int64_t cursor = a;
+    uint4 buf = make_uint4(0, 0, 0, 0);  // key of index cursor + lane
+    if (a + lane < b) buf = ld_nc_v4(keys + 32 * (a + lane));
+    for (;;) {
+        const uint32_t F = __ballot_sync(kFull, !busy);
+        if (F) {  // free lanes take the next keys, in lane order
+            const uint32_t rank = __popc(F & lanemask_lt());
+            const uint4 kin = shfl4(buf, rank);
+            if (!busy && cursor + rank < b) {
+                const int64_t e = cursor + rank;
+                if (is_zero(kin)) {  // the empty marker is never stored
+                    slots[e] = PK_NO_SLOT;
+                    first_miss = min(first_miss, (uint32_t)(e - a));
+                } else {
+                    probe_start(s, kin, (uint64_t)e, mask);
+                    busy = true;
+                }
+            }
+            const uint32_t nF = __popc(F);
+            buf = shfl4(buf, (lane + nF) & 31);
+            cursor += nF;
+            if (lane + nF >= 32 && cursor + lane < b) buf = ld_nc_v4(keys + 32 * (cursor + lane));
         }
-        const uint32_t ball = __ballot_sync(0xffffffffu, g < b && slot == PK_NO_SLOT);
-        if (h < 0 && ball) h = base - a + (__ffs(ball) - 1);
+        const uint32_t P = __ballot_sync(kFull, busy);
+        if (!P) {
+            if (cursor >= b) break;
+            continue;
+        }
+        uint32_t slot;
+        bool lim;
+        if (lookup_round(table, mask, max_probe, P, s, slot, lim)) {
+            slots[s.e] = slot;
+            if (slot == PK_NO_SLOT) first_miss = min(first_miss, (uint32_t)((int64_t)s.e - a));
+            limit |= lim;
+            busy = false;
+        }
     }
-    if (h < 0) h = b > a ? b - a : 0;
-    if (lane == 0) hit[r] = (int32_t)h;
+    const uint32_t h = __reduce_min_sync(kFull, first_miss);
+    if (lane == 0) hit[r] = h != 0xffffffffu ? (int32_t)h : (int32_t)(b > a ? b - a : 0);
     if (limit) set_status(status, PK_ERR_PROBE_LIMIT);
 }
 
-// One thread per key (few long requests): slots only; k_first_miss follows.
+// One warp per 32 consecutive keys (few long requests): slots only;
+// k_first_miss follows.
 __global__ void __launch_bounds__(256)
 k_lookup(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
          const uint8_t *__restrict__ keys, const int64_t *__restrict__ key_off, uint32_t R,
@@ -132,11 +290,29 @@ k_lookup(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
     pk::pdl_launch_dependents();
     pk::pdl_wait();
     const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (R == 0 || (uint64_t)g >= key_capacity || g >= __ldg(key_off + R)) return;
-    const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * g));
-    uint32_t slot;
-    if (!probe(table, mask, max_probe, key, slot)) set_status(status, PK_ERR_PROBE_LIMIT);
-    slots[g] = slot;
+    const int64_t total = R == 0 ? 0 : __ldg(key_off + R);
+    const int64_t end = total < (int64_t)key_capacity ? total : (int64_t)key_capacity;
+    if (g - (int64_t)(threadIdx.x & 31) >= end) return;  // uniform per warp
+    ProbeKey s;
+    s.pending = false;
+    uint32_t slot = PK_NO_SLOT;
+    bool limit = false;
+    if (g < end) {
+        const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * g));
+        if (!is_zero(key)) probe_start(s, key, (uint64_t)g, mask);  // the empty marker is never stored
+    }
+    for (;;) {
+        const uint32_t P = __ballot_sync(kFull, s.pending);
+        if (!P) break;
+        uint32_t sl;
+        bool lim;
+        if (lookup_round(table, mask, max_probe, P, s, sl, lim)) {
+            slot = sl;
+            limit = lim;
+        }
+    }
+    if (g < end) slots[g] = slot;
+    if (limit) set_status(status, PK_ERR_PROBE_LIMIT);
 }
 
 // One warp per request: h_r = index of the first PK_NO_SLOT among its keys.
@@ -155,7 +331,7 @@ k_first_miss(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capac
     for (int64_t base = a; base < b; base += 32) {
         const int64_t idx = base + lane;
         const bool miss = idx < b && __ldg(slots + idx) == PK_NO_SLOT;
-        const uint32_t ball = __ballot_sync(0xffffffffu, miss);
+        const uint32_t ball = __ballot_sync(kFull, miss);
         if (ball) {
             h = base - a + (__ffs(ball) - 1);
             break;
@@ -172,7 +348,7 @@ k_first_miss(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capac
 //   `owner` (atomicMax of ~index) and leave PENDING with the entry position
 //   in slot_out for kernel 2.
 // Capacity: when the table holds few enough entries that this call cannot
-// fill it (count + n < capacity), claims are counted once per warp at the
+// fill it (count + n < capacity), claims are counted once per block at the
 // end.  Otherwise a new key is refused (TABLE_FULL) once the count reaches
 // capacity - 1 and every claim is counted as it happens; claims racing at
 // that threshold can still take the last empty entries, after which probes
@@ -220,7 +396,7 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
             atomicMax(&ent->owner, me);
             res = PK_STORE_PENDING;
             out = (uint32_t)pos;
-            if (fast) return kClaimedHere;  // counted once per warp at the end
+            if (fast) return kClaimedHere;  // counted once per block at the end
             atomicAdd(counter, 1ull);
             return kDone;
         }
@@ -229,58 +405,175 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
     return kAdvance;
 }
 
-// Insert-if-absent of one entry (index e): result code, output slot/position,
-// and whether it claimed an entry that the caller must count (fast mode).
-__device__ __forceinline__ void claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
-                                      unsigned long long *counter, unsigned long long epoch, bool fast,
-                                      const uint4 &key, uint32_t my_slot, uint64_t e, int32_t &res, uint32_t &out,
-                                      bool &claimed_fast) {
-    out = PK_NO_SLOT;
-    claimed_fast = false;
-    if (is_zero(key)) {
-        res = PK_ERR_RESERVED_KEY;
-        return;
-    }
-    if (my_slot == PK_NO_SLOT) {
-        res = PK_ERR_ARG;
-        return;
-    }
-    const uint32_t me = ~(uint32_t)e;
-    const uint32_t win = mask + 1 < kWin ? (uint32_t)(mask + 1) : kWin;
-    const uint64_t pos = home_of(key) & mask;
-    uint64_t base = pos & ~(uint64_t)(win - 1);
-    uint32_t j0 = (uint32_t)(pos - base);
-    uint32_t probed = 0;
-    bool done = false;
-    res = PK_ERR_PROBE_LIMIT;
-    while (!done && probed < max_probe) {
-        pk_entry *grp = table + base;
+// An entry read as v can decide key k: it is empty, holds k, or is a torn
+// read of k being written (every word zero or k's).
+__device__ __forceinline__ bool may_decide(const uint4 &v, const uint4 &k) {
+    return (v.x == 0 || v.x == k.x) && (v.y == 0 || v.y == k.y) && (v.z == 0 || v.z == k.z) &&
+           (v.w == 0 || v.w == k.w);
+}
+
+// Where a table is shared by the claims of one store call.
+struct ClaimCtx {
+    pk_entry *table;
+    uint64_t mask;
+    uint32_t max_probe;
+    uint64_t capacity;
+    unsigned long long *counter;
+    unsigned long long epoch;
+    bool fast;
+};
+
+// Insert-if-absent: one round over the undecided keys P of the warp.
+// Returns true in the lanes whose key was decided in this round, with its
+// result code and output; `claims` counts the fast-mode claims this lane
+// made as decider (for any key of the warp).
+__device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, ProbeKey &s, int32_t &res,
+                                            uint32_t &out, uint32_t &claims) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t win = window_size(c.mask);
+    const bool full = P == kFull;  // as in lookup_round
+    const Round rd = full ? Round{1, 0, lane, true, 1u << lane, 1u << lane} : plan_round(P, lane);
+    const uint4 k = full ? s.key : shfl4(s.key, rd.owner);
+    const uint64_t wpos = full ? s.pos : __shfl_sync(kFull, s.pos, rd.owner);
+    const uint32_t wprobed = full ? s.probed : __shfl_sync(kFull, s.probed, rd.owner);
+    const uint64_t we = full ? s.e : __shfl_sync(kFull, s.e, rd.owner);
+    const uint64_t base0 = wpos & ~(uint64_t)(win - 1);
+    const uint32_t j0 = (uint32_t)(wpos - base0);
+    const uint64_t wb = (base0 + (uint64_t)rd.j * win) & c.mask;
+    int cand = -1;
+    uint32_t cseq = 0;
+    uint4 cv = make_uint4(0, 0, 0, 0);
+    if (rd.work) {
+        pk_entry *grp = c.table + wb;
         uint4 v[kWin];
 #pragma unroll
-        for (uint32_t u = 0; u < kWin; ++u)
-            if (u < win) v[u] = ld_volatile_v4(grp[u].k);
+        for (uint32_t u = 0; u < kWin; ++u) {  // entries before the sequence start are not read
+            v[u] = make_uint4(0, 0, 0, 0);
+            if (u < win && (rd.j > 0 || u >= j0)) v[u] = ld_volatile_v4(grp[u].k);
+        }
 #pragma unroll
         for (uint32_t u = 0; u < kWin; ++u) {
-            if (u < win && u >= j0 && !done && probed < max_probe) {
-                ++probed;
-                const Examine x = examine(grp + u, base + u, v[u], key, me, epoch, fast, counter, capacity, res, out);
-                if (x != kAdvance) done = true;
-                if (x == kClaimedHere) claimed_fast = true;
+            const uint32_t seq = rd.j * win + u - j0;
+            const bool in_seq = u < win && (rd.j > 0 || u >= j0) && wprobed + seq < c.max_probe;
+            if (in_seq && cand < 0 && may_decide(v[u], k)) {
+                cand = (int)u;
+                cseq = seq;
+                cv = v[u];
             }
         }
-        base = (base + win) & mask;
-        j0 = 0;
+    }
+    const uint32_t B = __ballot_sync(kFull, cand >= 0);
+    const bool decider = cand >= 0 && (B & rd.work_mask & lanemask_lt()) == 0;
+    int32_t dres = PK_ERR_PROBE_LIMIT;
+    uint32_t dout = PK_NO_SLOT;
+    bool dadv = false;
+    uint64_t dnext = 0;
+    uint32_t dprobed = 0;
+    if (decider) {
+        const uint64_t epos = wb + (uint32_t)cand;
+        const Examine x = examine(c.table + epos, epos, cv, k, ~(uint32_t)we, c.epoch, c.fast, c.counter, c.capacity,
+                                  dres, dout);
+        if (x == kClaimedHere) ++claims;
+        if (x == kAdvance) {  // lost the entry to a different key: continue after it
+            dadv = true;
+            dnext = (epos + 1) & c.mask;
+            dprobed = wprobed + cseq + 1;
+        }
+    }
+    const uint32_t ob = B & rd.own_mask;
+    int32_t g_res = dres;
+    uint32_t g_out = dout, g_probed = dprobed;
+    bool g_adv = dadv;
+    uint64_t g_next = dnext;
+    if (!full) {
+        const uint32_t src = ob ? __ffs(ob) - 1 : lane;
+        g_res = __shfl_sync(kFull, dres, src);
+        g_out = __shfl_sync(kFull, dout, src);
+        g_adv = __shfl_sync(kFull, (int)dadv, src) != 0;
+        g_next = __shfl_sync(kFull, dnext, src);
+        g_probed = __shfl_sync(kFull, dprobed, src);
+    }
+    if (!s.pending) return false;
+    if (ob && !g_adv) {
+        res = g_res;
+        out = g_out;
+        s.pending = false;
+        return true;
+    }
+    if (ob) {
+        s.pos = g_next;
+        s.probed = g_probed;
+    } else {
+        skip_windows(s, rd.G, win, c.mask);
+    }
+    if (s.probed >= c.max_probe) {
+        res = PK_ERR_PROBE_LIMIT;
+        out = PK_NO_SLOT;
+        s.pending = false;
+        return true;
+    }
+    return false;
+}
+
+// Insert-if-absent of at most one key per lane, all lanes together.
+__device__ __forceinline__ void warp_claim(const ClaimCtx &c, ProbeKey &s, int32_t &res, uint32_t &out,
+                                           uint32_t &claims) {
+    for (;;) {
+        const uint32_t P = __ballot_sync(kFull, s.pending);
+        if (!P) break;
+        claim_round(c, P, s, res, out, claims);
     }
 }
 
-// List mode, or range mode for few long requests: one thread per entry.
-__global__ void __launch_bounds__(256)
+// Argument checks of one entry before it is claimed: a zero key is the
+// empty marker; PK_NO_SLOT is not a storable slot.
+__device__ __forceinline__ bool claimable(const uint4 &key, uint32_t slot, int32_t &res) {
+    if (is_zero(key)) {
+        res = PK_ERR_RESERVED_KEY;
+        return false;
+    }
+    if (slot == PK_NO_SLOT) {
+        res = PK_ERR_ARG;
+        return false;
+    }
+    return true;
+}
+
+// Whether entry e lies in the store range of its request, [key_off[r] + h_r,
+// key_off[r+1]) (range mode; warp-collective).
+__device__ __forceinline__ bool in_store_range(const int64_t *__restrict__ key_off, const int32_t *__restrict__ hit,
+                                               uint32_t R, uint64_t n, uint64_t e) {
+    const uint64_t e0 = e - (threadIdx.x & 31);
+    const int64_t total = R > 0 ? __ldg(key_off + R) : 0;
+    bool in_range = false;
+    if (e0 < n && (int64_t)e0 < total) {
+        const uint32_t r = pk::lane_request(key_off, R, (int64_t)e0, total, (int64_t)e);
+        if ((int64_t)e < total) {
+            const int64_t h = __ldg(hit + r);
+            in_range = (int64_t)e - __ldg(key_off + r) >= (h > 0 ? h : 0);
+        }
+    }
+    return in_range;
+}
+
+// Adds the warp's fast-mode claims to the block total, then the block total
+// to the entry counter (same-address atomics serialise in L2).
+__device__ __forceinline__ void count_claims(unsigned long long *block_claims, uint32_t claims,
+                                             unsigned long long *counter) {
+    const uint32_t w = __reduce_add_sync(kFull, claims);
+    if ((threadIdx.x & 31) == 0 && w) atomicAdd_block(block_claims, (unsigned long long)w);
+    __syncthreads();
+    if (threadIdx.x == 0 && *block_claims) atomicAdd(counter, *block_claims);
+}
+
+// List mode, or range mode for few long requests: one warp per 32
+// consecutive entries.
+__global__ void __launch_bounds__(256, 4)
 k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
               unsigned long long *counter, unsigned long long epoch, const uint8_t *__restrict__ keys,
               const uint32_t *__restrict__ slots, uint64_t n, const int64_t *__restrict__ key_off,
               const int32_t *__restrict__ hit, uint32_t R, int32_t *__restrict__ result,
               uint32_t *__restrict__ slot_out, int32_t *status) {
-    // Claims are counted once per block: same-address atomics serialise in L2.
     __shared__ unsigned long long block_claims;
     if (threadIdx.x == 0) block_claims = 0;
     __syncthreads();
@@ -288,51 +581,40 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
     pk::pdl_wait();
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const uint32_t lane = threadIdx.x & 31;
-    const uint64_t e0 = e - lane;
     bool active = e < n;
-    if (key_off) {  // range mode: only [key_off[r] + hit[r], key_off[r+1])
-        const int64_t total = R > 0 ? __ldg(key_off + R) : 0;
-        bool in_range = false;
-        if (e0 < n && (int64_t)e0 < total) {
-            const uint32_t r = pk::lane_request(key_off, R, (int64_t)e0, total, (int64_t)e);
-            if ((int64_t)e < total) {
-                const int64_t h = __ldg(hit + r);
-                in_range = (int64_t)e - __ldg(key_off + r) >= (h > 0 ? h : 0);
-            }
-        }
-        active = active && in_range;
-    }
+    if (key_off) active = in_store_range(key_off, hit, R, n, e) && active;
     unsigned long long cnt = 0;
     if (lane == 0) cnt = ld_volatile_u64(counter);
-    const bool fast = __shfl_sync(0xffffffffu, cnt, 0) + n < capacity;
+    const bool fast = __shfl_sync(kFull, cnt, 0) + n < capacity;
+    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast};
     int32_t res = PK_STORE_SKIPPED;
     uint32_t out = PK_NO_SLOT;
-    bool claimed_fast = false;
+    ProbeKey s;
+    s.pending = false;
     if (active) {
         const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
-        claim(table, mask, max_probe, capacity, counter, epoch, fast, key, slots[e], e, res, out, claimed_fast);
+        if (claimable(key, slots[e], res)) probe_start(s, key, e, mask);
     }
+    uint32_t claims = 0;
+    warp_claim(c, s, res, out, claims);
     if (e < n) {
         result[e] = res;
         slot_out[e] = out;
         if (res < 0) set_status(status, res);
     }
-    const uint32_t m = __ballot_sync(0xffffffffu, claimed_fast);
-    if (lane == 0 && m) atomicAdd_block(&block_claims, (unsigned long long)__popc(m));
-    __syncthreads();
-    if (threadIdx.x == 0 && block_claims) atomicAdd(counter, block_claims);
+    count_claims(&block_claims, claims, counter);
 }
 
 // Range mode for many short requests: one warp per request, no search.
 // Writes every entry of [key_off[r], key_off[r+1]); entries past key_off[R]
 // are marked by the finalize kernel.
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(256, 4)
 k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
                   unsigned long long *counter, unsigned long long epoch, const uint8_t *__restrict__ keys,
                   const uint32_t *__restrict__ slots, uint64_t n, const int64_t *__restrict__ key_off,
                   const int32_t *__restrict__ hit, uint32_t R, int32_t *__restrict__ result,
                   uint32_t *__restrict__ slot_out, int32_t *status) {
-    __shared__ unsigned long long block_claims;  // counted once per block (see k_store_claim)
+    __shared__ unsigned long long block_claims;
     if (threadIdx.x == 0) block_claims = 0;
     __syncthreads();
     pk::pdl_launch_dependents();
@@ -349,28 +631,65 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
     }
     unsigned long long cnt = 0;
     if (lane == 0) cnt = ld_volatile_u64(counter);
-    const bool fast = __shfl_sync(0xffffffffu, cnt, 0) + n < capacity;
-    uint32_t claimed = 0;
-    for (int64_t base = a; base < b; base += 32) {
-        const int64_t e = base + lane;
-        int32_t res = PK_STORE_SKIPPED;
-        uint32_t out = PK_NO_SLOT;
-        bool claimed_fast = false;
-        if (e < b && e >= first) {
-            const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
-            claim(table, mask, max_probe, capacity, counter, epoch, fast, key, slots[e], (uint64_t)e, res, out,
-                  claimed_fast);
+    const bool fast = __shfl_sync(kFull, cnt, 0) + n < capacity;
+    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast};
+    uint32_t claims = 0;
+    for (int64_t x = a + lane; x < first && x < b; x += 32) {  // below h_r: not stored
+        result[x] = PK_STORE_SKIPPED;
+        slot_out[x] = PK_NO_SLOT;
+    }
+    // The store range [first, b): a lane whose key is decided takes the next
+    // one from a register buffer of the next 32 keys and slots (as in
+    // k_lookup_req).
+    ProbeKey s;
+    s.pending = false;
+    int64_t cursor = first;
+    uint4 buf = make_uint4(0, 0, 0, 0);  // key and slot of index cursor + lane
+    uint32_t buf_slot = 0;
+    if (first + lane < b) {
+        buf = ld_nc_v4(keys + 32 * (first + lane));
+        buf_slot = __ldg(slots + first + lane);
+    }
+    for (;;) {
+        const uint32_t F = __ballot_sync(kFull, !s.pending);
+        if (F) {  // free lanes take the next keys, in lane order
+            const uint32_t rank = __popc(F & lanemask_lt());
+            const uint4 kin = shfl4(buf, rank);
+            const uint32_t sin = __shfl_sync(kFull, buf_slot, rank);
+            if (!s.pending && cursor + rank < b) {
+                const int64_t e = cursor + rank;
+                int32_t res;
+                if (claimable(kin, sin, res)) {
+                    probe_start(s, kin, (uint64_t)e, mask);
+                } else {
+                    result[e] = res;
+                    slot_out[e] = PK_NO_SLOT;
+                    set_status(status, res);
+                }
+            }
+            const uint32_t nF = __popc(F);
+            buf = shfl4(buf, (lane + nF) & 31);
+            buf_slot = __shfl_sync(kFull, buf_slot, (lane + nF) & 31);
+            cursor += nF;
+            if (lane + nF >= 32 && cursor + lane < b) {
+                buf = ld_nc_v4(keys + 32 * (cursor + lane));
+                buf_slot = __ldg(slots + cursor + lane);
+            }
         }
-        if (e < b) {
-            result[e] = res;
-            slot_out[e] = out;
+        const uint32_t P = __ballot_sync(kFull, s.pending);
+        if (!P) {
+            if (cursor >= b) break;
+            continue;
+        }
+        int32_t res;
+        uint32_t out;
+        if (claim_round(c, P, s, res, out, claims)) {
+            result[s.e] = res;
+            slot_out[s.e] = out;
             if (res < 0) set_status(status, res);
         }
-        claimed += __popc(__ballot_sync(0xffffffffu, claimed_fast));
     }
-    if (lane == 0 && claimed) atomicAdd_block(&block_claims, (unsigned long long)claimed);
-    __syncthreads();
-    if (threadIdx.x == 0 && block_claims) atomicAdd(counter, block_claims);
+    count_claims(&block_claims, claims, counter);
 }
 
 // Store, kernel 2 of 2: the lowest claimant of each new key writes its slot.
@@ -450,9 +769,10 @@ k_noalloc_scan(const pk_entry *__restrict__ table, uint64_t capacity, NoallocScr
     }
 }
 
-// One thread per entry (list or range mode), as k_store_claim; the call
-// number is one past the table's latest and PENDING positions go to scratch.
-__global__ void __launch_bounds__(256)
+// One warp per 32 consecutive entries (list or range mode), as
+// k_store_claim; the call number is one past the table's latest and PENDING
+// positions go to scratch.
+__global__ void __launch_bounds__(256, 4)
 k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity, NoallocScratch *sc,
                 const uint8_t *__restrict__ keys, const uint32_t *__restrict__ slots, uint64_t n,
                 const int64_t *__restrict__ key_off, const int32_t *__restrict__ hit, uint32_t R,
@@ -463,30 +783,22 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
     const unsigned long long epoch = ld_volatile_u64(&sc->epoch_max) + 1ull;
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const uint32_t lane = threadIdx.x & 31;
-    const uint64_t e0 = e - lane;
     bool active = e < n;
-    if (key_off) {
-        const int64_t total = R > 0 ? __ldg(key_off + R) : 0;
-        bool in_range = false;
-        if (e0 < n && (int64_t)e0 < total) {
-            const uint32_t r = pk::lane_request(key_off, R, (int64_t)e0, total, (int64_t)e);
-            if ((int64_t)e < total) {
-                const int64_t h = __ldg(hit + r);
-                in_range = (int64_t)e - __ldg(key_off + r) >= (h > 0 ? h : 0);
-            }
-        }
-        active = active && in_range;
-    }
+    if (key_off) active = in_store_range(key_off, hit, R, n, e) && active;
     unsigned long long cnt = 0;
     if (lane == 0) cnt = ld_volatile_u64(&sc->count);
-    const bool fast = __shfl_sync(0xffffffffu, cnt, 0) + n < capacity;
+    const bool fast = __shfl_sync(kFull, cnt, 0) + n < capacity;
+    const ClaimCtx c{table, mask, max_probe, capacity, &sc->count, epoch, fast};
     int32_t res = PK_STORE_SKIPPED;
     uint32_t out = PK_NO_SLOT;
-    bool claimed_fast = false;
+    ProbeKey s;
+    s.pending = false;
     if (active) {
         const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
-        claim(table, mask, max_probe, capacity, &sc->count, epoch, fast, key, slots[e], e, res, out, claimed_fast);
+        if (claimable(key, slots[e], res)) probe_start(s, key, e, mask);
     }
+    uint32_t claims = 0;
+    warp_claim(c, s, res, out, claims);
     if (e < n) {
         result[e] = res;
         if (res == PK_STORE_PENDING) {
@@ -497,10 +809,7 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
         }
         if (res < 0) set_status(status, res);
     }
-    const uint32_t m = __ballot_sync(0xffffffffu, claimed_fast);
-    if (lane == 0 && m) atomicAdd_block(&block_claims, (unsigned long long)__popc(m));
-    __syncthreads();
-    if (threadIdx.x == 0 && block_claims) atomicAdd(&sc->count, block_claims);
+    count_claims(&block_claims, claims, &sc->count);
 }
 
 __global__ void __launch_bounds__(256)
