@@ -6,6 +6,7 @@ One step = one pass of the whole hot path over one batch:
   a0  canonicalise + encode the batch's descriptors (host), SHA-256 -> d (device)
   a1  chunk digests c_i          a2  chained keys k_i
   a3  probe every key            a4  store the miss ranges
+(a3 and a4 in one pass: pk_lookup_store).
 Default workload: the multi-adapter serving configuration (1024 requests x
 4096 tokens, chunk 256, 32 descriptors, table of 2^20 entries at load 0.5).
 
@@ -303,9 +304,8 @@ def main():
         pk.pk_derive_keys_enc(ctx, tokens_d, tok_off_d, desc_idx_d, enc_h[:n_enc], enc_off_h, digests_d, key_off_d,
                               keys_d, status)
         if ev: ev[2].record(stream)
-        pk.pk_lookup(ctx, keys_d, key_off_d, hit_d, slots_d, status)           # a3
-        if ev: ev[3].record(stream)
-        pk.pk_store(ctx, keys_d, new_slots_d, result_d, slot_out_d, status, key_off_d, hit_d)  # a4
+        # a3 (lookup as of the start of the call) and a4 (store of the miss ranges) in one pass
+        pk.pk_lookup_store(ctx, keys_d, new_slots_d, key_off_d, hit_d, slots_d, result_d, slot_out_d, status)
 
     def between_steps():
         kt.load(snapshot)
@@ -322,26 +322,26 @@ def main():
     if kt.take_status() != 0:
         raise RuntimeError("device status after warm-up")
     hit_ref = hit_d.cpu().numpy().copy()
+    inserted = kt.entries() - wl.target_entries  # keys one step inserts (the table is restored between steps)
 
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
     clocks.start()
-    step_ms, derive_ms, lookup_ms, store_ms, a0_ms = [], [], [], [], []
+    step_ms, derive_ms, table_ms, a0_ms = [], [], [], []
     for _ in range(args.steps):
         between_steps()
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
         torch.cuda._sleep(spin_cycles)
         ev[0].record(stream)
         core(ev)
-        ev[4].record(stream)
+        ev[3].record(stream)
         torch.cuda.synchronize()
-        step_ms.append(ev[0].elapsed_time(ev[4]))
+        step_ms.append(ev[0].elapsed_time(ev[3]))
         a0_ms.append(ev[0].elapsed_time(ev[1]))
         derive_ms.append(ev[1].elapsed_time(ev[2]))
-        lookup_ms.append(ev[2].elapsed_time(ev[3]))
-        store_ms.append(ev[3].elapsed_time(ev[4]))
+        table_ms.append(ev[2].elapsed_time(ev[3]))
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
@@ -360,8 +360,8 @@ def main():
             pk.pk_descriptors_encode(descs, enc_h.numpy(), enc_off_h.numpy())
             pk.pk_derive_keys_enc(ctx, tokens_h, tok_off_h, desc_idx_h, enc_h[:n_enc], enc_off_h, digests_d,
                                   key_off_d, keys_d, status)
-            pk.pk_lookup(ctx, keys_d, key_off_d, hit_d, slots_d, status)
-            pk.pk_store(ctx, keys_d, new_slots_d, result_d, slot_out_d, status, key_off_d, hit_d)
+            pk.pk_lookup_store(ctx, keys_d, new_slots_d, key_off_d, hit_d, slots_d, result_d, slot_out_d,
+                               status)
         else:
             tokens_d.copy_(tokens_h, non_blocking=True)
             tok_off_d.copy_(tok_off_h, non_blocking=True)
@@ -411,8 +411,10 @@ def main():
     # schedule word): the ceiling for this formulation, in the same 1384-op units
     alu_pipe_peak = SMS * 64 * peaks["sm_max_mhz"] * 1e6 / 1024 * SHA_OPS_PER_COMPRESSION / 1e12
     achieved = (c_dig + c_chain) * SHA_OPS_PER_COMPRESSION / derive_s / 1e12
-    lookup_s = float(np.mean(lookup_ms)) / 1e3
-    probe_bytes = n_keys * (16 + 32 + 4) + R * 4
+    table_s = float(np.mean(table_ms)) / 1e3
+    # per key: 16 B key + one 32 B entry sector + 4 B new slot + 12 B of outputs (lookup slot, result,
+    # output slot); per inserted key one 32 B entry sector written; 4 B (h_r) per request
+    probe_bytes = n_keys * (16 + 32 + 4 + 12) + inserted * 32 + R * 4
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
@@ -421,7 +423,8 @@ def main():
         "lookups_per_s": n_keys * args.steps * world / (total_ms / 1e3),
         "requests_per_s": R * args.steps * world / (total_ms / 1e3),
         "phase_ms": {"a0_host": float(np.mean(a0_ms)), "descriptors_and_keys": float(np.mean(derive_ms)),
-                     "lookup": float(np.mean(lookup_ms)), "store": float(np.mean(store_ms))},
+                     "lookup_and_store": float(np.mean(table_ms))},
+        "inserted_per_step": inserted,
         "roofline": {"bound": "alu",
                      "kernel": "pk_derive_keys_enc (chunk offsets; chunk + descriptor digests; chain)",
                      "achieved": achieved, "peak": alu_peak, "unit": "Tops/s", "frac": achieved / alu_peak,
@@ -431,10 +434,11 @@ def main():
                      "peak_basis": f"{SMS} SMs x {LANES_PER_SM} int32 lanes x {peaks['sm_max_mhz']:.0f} MHz "
                                    f"(issue-rate ceiling); {SHA_OPS_PER_COMPRESSION} ops per compression, "
                                    f"{c_dig + c_chain} compressions per launch"},
-        "probe_roofline": {"bound": "hbm", "kernel": "pk_lookup", "achieved": probe_bytes / lookup_s / 1e9,
-                           "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                           "frac": probe_bytes / lookup_s / 1e9 / peaks["hbm_gbs"],
-                           "bytes_basis": "per probe 16 B key + one 32 B entry sector + 4 B slot; 4 B per request",
+        "probe_roofline": {"bound": "hbm", "kernel": "pk_lookup_store (probe + claim; finalize)",
+                           "achieved": probe_bytes / table_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                           "frac": probe_bytes / table_s / 1e9 / peaks["hbm_gbs"],
+                           "bytes_basis": "per key 16 B key + one 32 B entry sector + 4 B new slot + 12 B "
+                                          "outputs; 32 B per inserted key; 4 B per request",
                            "peak_source": peaks["source"]},
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_total / args.steps,
@@ -443,9 +447,9 @@ def main():
                 "in_place_reads": {"value": tokens_per_step * args.steps * world / (e2e_inplace_total / 1e3),
                                    "ms_per_step": e2e_inplace_total / args.steps,
                                    "note": "all inputs read by the kernels from pinned host memory"}},
-        # per step: chunk offsets, chunk+descriptor digests, chain; lookup (one kernel per request
-        # warp, or per key + first miss for few long requests); store claim + finalize
-        "gpu_launches": (3 + (1 if (R >= 1024 or N_cap <= 64 * R) else 2) + 2) * args.steps,
+        # per step: chunk offsets, chunk+descriptor digests, chain; lookup-and-store (one kernel of
+        # request warps, or per key + per-request tail for few long requests); finalize
+        "gpu_launches": (3 + (1 if (R >= 1024 or N_cap <= 64 * R) else 2) + 1) * args.steps,
         "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -205,6 +205,26 @@ int pk_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_dev, ui
              const int64_t *key_off_dev, const int32_t *hit_chunks_dev, uint32_t R,
              int32_t *result_dev, uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream);
 
+/* Device.  pk_lookup followed by pk_store in range mode, in one pass over
+ * the keys (Sec. 2.1: the connector looks the chunks up, and a miss computes
+ * and writes new state).  Every key of the batch is inserted if absent, keys
+ * inserted earlier in the same call counting as absent, so each key's probe
+ * sequence is walked once:
+ *   slots_dev, hit_chunks_dev  OUT as pk_lookup (the table as of the start
+ *                              of the call)
+ *   result_dev, slot_out_dev   OUT as pk_store in range mode over the miss
+ *                              ranges [key_off[r] + h_r, key_off[r+1]) with
+ *                              slots slots_new_dev; other entries
+ *                              PK_STORE_SKIPPED
+ * keys_dev as pk_lookup (16-byte aligned); slots_new_dev, slots_dev,
+ * result_dev, slot_out_dev: key_capacity entries of 4 bytes.  A key whose new
+ * slot is PK_NO_SLOT is only looked up (PK_ERR_ARG if it lies in its miss
+ * range).  Results equal those of the two calls; device errors as the two
+ * calls, the first one observed going to *status_dev. */
+int pk_lookup_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_new_dev, const int64_t *key_off_dev,
+                    uint32_t R, uint64_t key_capacity, int32_t *hit_chunks_dev, uint32_t *slots_dev,
+                    int32_t *result_dev, uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream);
+
 /* Checkpoint (the shared store outlives workers, Sec. 2.1).  Asynchronous on
  * `stream`: copies the table and its entry count to dst (device or host
  * memory, dst_bytes >= pk_table_bytes(capacity_log2) + 64). */

@@ -244,6 +244,24 @@ int pk_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_dev, ui
                                    reinterpret_cast<cudaStream_t>(stream)));
 }
 
+int pk_lookup_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_new_dev, const int64_t *key_off_dev,
+                    uint32_t R, uint64_t key_capacity, int32_t *hit_chunks_dev, uint32_t *slots_dev,
+                    int32_t *result_dev, uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream) {
+    if (!ctx || !key_off_dev) return PK_ERR_ARG;
+    if (R && !hit_chunks_dev) return PK_ERR_ARG;
+    if (key_capacity &&
+        (!keys_dev || !aligned16(keys_dev) || !slots_new_dev || !slots_dev || !result_dev || !slot_out_dev))
+        return PK_ERR_ARG;
+    if (key_capacity > (uint64_t)0x7fffffff * 256 || key_capacity >= 0xffffffffull) return PK_ERR_ARG;
+    if (!aligned(key_off_dev, 8) || !aligned(hit_chunks_dev, 4) || !aligned(slots_new_dev, 4) ||
+        !aligned(slots_dev, 4) || !aligned(result_dev, 4) || !aligned(slot_out_dev, 4))
+        return PK_ERR_ARG;
+    const unsigned long long epoch = ++ctx->epoch;
+    return cuda_rc(pk_launch_lookup_store(ctx, epoch, keys_dev, slots_new_dev, key_off_dev, R, key_capacity,
+                                          hit_chunks_dev, slots_dev, result_dev, slot_out_dev, status_dev,
+                                          reinterpret_cast<cudaStream_t>(stream)));
+}
+
 int pk_table_save(pk_ctx *ctx, void *dst, size_t dst_bytes, pk_stream stream) {
     if (!ctx || !dst) return PK_ERR_ARG;
     const size_t tb = pk_table_bytes(ctx->capacity_log2);

@@ -135,14 +135,17 @@ struct ProbeKey {
     uint64_t pos;     // next table position of its probe sequence
     uint32_t probed;  // entries of the sequence examined so far
     bool pending;     // not decided yet
+    bool may_claim;   // lookup-and-store: the key may be inserted (its slot is valid)
 };
 
-__device__ __forceinline__ void probe_start(ProbeKey &s, const uint4 &key, uint64_t e, uint64_t mask) {
+__device__ __forceinline__ void probe_start(ProbeKey &s, const uint4 &key, uint64_t e, uint64_t mask,
+                                            bool may_claim = true) {
     s.key = key;
     s.e = e;
     s.pos = home_of(key) & mask;
     s.probed = 0;
     s.pending = true;
+    s.may_claim = may_claim;
 }
 
 // Owner role after a round in which no lane of its group found a deciding
@@ -357,10 +360,17 @@ k_first_miss(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capac
 enum Examine { kAdvance, kDone, kClaimedHere };
 
 // Examine entry `ent` (position pos) whose key was read as `cur`.
+// kFused (lookup-and-store): `present` tells whether the key was in the
+// table when the call started (inserted by an earlier call: epoch set and
+// not this call's), with its slot in lslot; a key that may not be inserted
+// (!may_claim) ends with PK_ERR_ARG and leaves the table untouched.
+template <bool kFused>
 __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cur, const uint4 &key, uint32_t me,
                                            unsigned long long epoch, bool fast, unsigned long long *counter,
-                                           uint64_t capacity, int32_t &res, uint32_t &out) {
+                                           uint64_t capacity, bool may_claim, int32_t &res, uint32_t &out,
+                                           uint32_t &lslot) {
     uint4 *kp = reinterpret_cast<uint4 *>(ent->k);
+    lslot = PK_NO_SLOT;
 #pragma unroll 1
     for (int pass = 0; pass < 2; ++pass) {
         // A vector load racing a concurrent 128-bit CAS may observe a mix of
@@ -373,16 +383,26 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
         if (same(cur, key)) {
             const unsigned long long ep = ld_volatile_u64(&ent->epoch);
             if (ep != 0ull && ep != epoch) {  // inserted by an earlier call
-                res = PK_STORE_PRESENT;
-                out = *(volatile uint32_t *)&ent->slot;
-            } else {  // claimed during this call
+                const uint32_t sl = *(volatile uint32_t *)&ent->slot;
+                if (kFused) lslot = sl;
+                res = (!kFused || may_claim) ? PK_STORE_PRESENT : PK_ERR_ARG;
+                out = (!kFused || may_claim) ? sl : PK_NO_SLOT;
+            } else if (!kFused || may_claim) {  // claimed during this call
                 atomicMax(&ent->owner, me);
                 res = PK_STORE_PENDING;
                 out = (uint32_t)pos;
+            } else {
+                res = PK_ERR_ARG;
+                out = PK_NO_SLOT;
             }
             return kDone;
         }
         if (!is_zero(cur)) return kAdvance;  // a different key holds this entry
+        if (kFused && !may_claim) {          // absent; not to be inserted
+            res = PK_ERR_ARG;
+            out = PK_NO_SLOT;
+            return kDone;
+        }
         // Room check: refuse a new key once the table holds capacity - 1
         // entries.  Only successful claims are counted (below), so racing
         // duplicates of one key never touch the counter.
@@ -427,8 +447,11 @@ struct ClaimCtx {
 // Returns true in the lanes whose key was decided in this round, with its
 // result code and output; `claims` counts the fast-mode claims this lane
 // made as decider (for any key of the warp).
+// kFused: also `lslot`, the key's slot if it was in the table when the call
+// started (else PK_NO_SLOT), and keys with !may_claim are looked up only.
+template <bool kFused>
 __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, ProbeKey &s, int32_t &res,
-                                            uint32_t &out, uint32_t &claims) {
+                                            uint32_t &out, uint32_t &lslot, uint32_t &claims) {
     const uint32_t lane = threadIdx.x & 31;
     const uint32_t win = window_size(c.mask);
     const bool full = P == kFull;  // as in lookup_round
@@ -437,6 +460,7 @@ __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, Probe
     const uint64_t wpos = full ? s.pos : __shfl_sync(kFull, s.pos, rd.owner);
     const uint32_t wprobed = full ? s.probed : __shfl_sync(kFull, s.probed, rd.owner);
     const uint64_t we = full ? s.e : __shfl_sync(kFull, s.e, rd.owner);
+    const bool wmay = !kFused || (full ? s.may_claim : __shfl_sync(kFull, (int)s.may_claim, rd.owner) != 0);
     const uint64_t base0 = wpos & ~(uint64_t)(win - 1);
     const uint32_t j0 = (uint32_t)(wpos - base0);
     const uint64_t wb = (base0 + (uint64_t)rd.j * win) & c.mask;
@@ -465,14 +489,14 @@ __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, Probe
     const uint32_t B = __ballot_sync(kFull, cand >= 0);
     const bool decider = cand >= 0 && (B & rd.work_mask & lanemask_lt()) == 0;
     int32_t dres = PK_ERR_PROBE_LIMIT;
-    uint32_t dout = PK_NO_SLOT;
+    uint32_t dout = PK_NO_SLOT, dls = PK_NO_SLOT;
     bool dadv = false;
     uint64_t dnext = 0;
     uint32_t dprobed = 0;
     if (decider) {
         const uint64_t epos = wb + (uint32_t)cand;
-        const Examine x = examine(c.table + epos, epos, cv, k, ~(uint32_t)we, c.epoch, c.fast, c.counter, c.capacity,
-                                  dres, dout);
+        const Examine x = examine<kFused>(c.table + epos, epos, cv, k, ~(uint32_t)we, c.epoch, c.fast, c.counter,
+                                          c.capacity, wmay, dres, dout, dls);
         if (x == kClaimedHere) ++claims;
         if (x == kAdvance) {  // lost the entry to a different key: continue after it
             dadv = true;
@@ -482,13 +506,14 @@ __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, Probe
     }
     const uint32_t ob = B & rd.own_mask;
     int32_t g_res = dres;
-    uint32_t g_out = dout, g_probed = dprobed;
+    uint32_t g_out = dout, g_probed = dprobed, g_ls = dls;
     bool g_adv = dadv;
     uint64_t g_next = dnext;
     if (!full) {
         const uint32_t src = ob ? __ffs(ob) - 1 : lane;
         g_res = __shfl_sync(kFull, dres, src);
         g_out = __shfl_sync(kFull, dout, src);
+        if (kFused) g_ls = __shfl_sync(kFull, dls, src);
         g_adv = __shfl_sync(kFull, (int)dadv, src) != 0;
         g_next = __shfl_sync(kFull, dnext, src);
         g_probed = __shfl_sync(kFull, dprobed, src);
@@ -497,6 +522,7 @@ __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, Probe
     if (ob && !g_adv) {
         res = g_res;
         out = g_out;
+        lslot = g_ls;
         s.pending = false;
         return true;
     }
@@ -509,19 +535,22 @@ __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, Probe
     if (s.probed >= c.max_probe) {
         res = PK_ERR_PROBE_LIMIT;
         out = PK_NO_SLOT;
+        lslot = PK_NO_SLOT;
         s.pending = false;
         return true;
     }
     return false;
 }
 
-// Insert-if-absent of at most one key per lane, all lanes together.
+// Insert-if-absent (kFused: lookup-and-store) of at most one key per lane,
+// all lanes together.
+template <bool kFused>
 __device__ __forceinline__ void warp_claim(const ClaimCtx &c, ProbeKey &s, int32_t &res, uint32_t &out,
-                                           uint32_t &claims) {
+                                           uint32_t &lslot, uint32_t &claims) {
     for (;;) {
         const uint32_t P = __ballot_sync(kFull, s.pending);
         if (!P) break;
-        claim_round(c, P, s, res, out, claims);
+        claim_round<kFused>(c, P, s, res, out, lslot, claims);
     }
 }
 
@@ -595,8 +624,8 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
         const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
         if (claimable(key, slots[e], res)) probe_start(s, key, e, mask);
     }
-    uint32_t claims = 0;
-    warp_claim(c, s, res, out, claims);
+    uint32_t claims = 0, lslot;
+    warp_claim<false>(c, s, res, out, lslot, claims);
     if (e < n) {
         result[e] = res;
         slot_out[e] = out;
@@ -682,14 +711,197 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
             continue;
         }
         int32_t res;
-        uint32_t out;
-        if (claim_round(c, P, s, res, out, claims)) {
+        uint32_t out, lslot;
+        if (claim_round<false>(c, P, s, res, out, lslot, claims)) {
             result[s.e] = res;
             slot_out[s.e] = out;
             if (res < 0) set_status(status, res);
         }
     }
     count_claims(&block_claims, claims, counter);
+}
+
+// ---------------------------------------------------------------------------
+// Lookup and store in one pass (pk_lookup_store).  Every key of the batch is
+// inserted if absent, and keys inserted earlier in the same call count as
+// absent: a key inserted by an earlier call is a hit (with its slot), any
+// other key a miss.  That is the lookup of the table as of the start of the
+// call.  h_r is the first miss of request r and every miss lies at or after
+// h_r, so the insertions made are exactly those of storing [h_r, n_r) after
+// the lookup; the entries below h_r (all hits) are then relabelled
+// PK_STORE_SKIPPED.  A key whose slot is PK_NO_SLOT is only looked up and
+// ends with PK_ERR_ARG when it lies in the store range.
+// ---------------------------------------------------------------------------
+
+// One warp per request, refilled from a register buffer as k_lookup_req.
+__global__ void __launch_bounds__(256, 3)
+k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
+                   unsigned long long *counter, unsigned long long epoch, const uint8_t *__restrict__ keys,
+                   const uint32_t *__restrict__ new_slots, const int64_t *__restrict__ key_off, uint32_t R,
+                   uint64_t key_capacity, uint32_t *__restrict__ slots, int32_t *__restrict__ hit,
+                   int32_t *__restrict__ result, uint32_t *__restrict__ slot_out, int32_t *status) {
+    __shared__ unsigned long long block_claims;
+    if (threadIdx.x == 0) block_claims = 0;
+    __syncthreads();
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
+    const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const uint32_t lane = threadIdx.x & 31;
+    int64_t a = 0, b = 0;
+    if (r < R) {  // uniform per warp
+        a = __ldg(key_off + r);
+        b = __ldg(key_off + r + 1);
+        if ((uint64_t)b > key_capacity) b = (int64_t)key_capacity;
+    }
+    unsigned long long cnt = 0;
+    if (lane == 0) cnt = ld_volatile_u64(counter);
+    const bool fast = __shfl_sync(kFull, cnt, 0) + key_capacity < capacity;
+    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast};
+    uint32_t claims = 0;
+    uint32_t first_miss = 0xffffffffu;  // lowest miss index (relative to a) seen by this lane
+    int64_t arg_hit = -1;               // highest index of a hit whose slot was PK_NO_SLOT
+    ProbeKey s;
+    s.pending = false;
+    int64_t cursor = a;
+    uint4 buf = make_uint4(0, 0, 0, 0);  // key and slot of index cursor + lane
+    uint32_t buf_slot = 0;
+    if (a + lane < b) {
+        buf = ld_nc_v4(keys + 32 * (a + lane));
+        buf_slot = __ldg(new_slots + a + lane);
+    }
+    for (;;) {
+        const uint32_t F = __ballot_sync(kFull, !s.pending);
+        if (F) {  // free lanes take the next keys, in lane order
+            const uint32_t rank = __popc(F & lanemask_lt());
+            const uint4 kin = shfl4(buf, rank);
+            const uint32_t sin = __shfl_sync(kFull, buf_slot, rank);
+            if (!s.pending && cursor + rank < b) {
+                const int64_t e = cursor + rank;
+                if (is_zero(kin)) {  // the empty marker: never stored, so a miss
+                    slots[e] = PK_NO_SLOT;
+                    result[e] = PK_ERR_RESERVED_KEY;
+                    slot_out[e] = PK_NO_SLOT;
+                    set_status(status, PK_ERR_RESERVED_KEY);
+                    first_miss = min(first_miss, (uint32_t)(e - a));
+                } else {
+                    probe_start(s, kin, (uint64_t)e, mask, sin != PK_NO_SLOT);
+                }
+            }
+            const uint32_t nF = __popc(F);
+            buf = shfl4(buf, (lane + nF) & 31);
+            buf_slot = __shfl_sync(kFull, buf_slot, (lane + nF) & 31);
+            cursor += nF;
+            if (lane + nF >= 32 && cursor + lane < b) {
+                buf = ld_nc_v4(keys + 32 * (cursor + lane));
+                buf_slot = __ldg(new_slots + cursor + lane);
+            }
+        }
+        const uint32_t P = __ballot_sync(kFull, s.pending);
+        if (!P) {
+            if (cursor >= b) break;
+            continue;
+        }
+        int32_t res;
+        uint32_t out, lslot;
+        if (claim_round<true>(c, P, s, res, out, lslot, claims)) {
+            const int64_t e = (int64_t)s.e;
+            slots[e] = lslot;
+            result[e] = res;
+            slot_out[e] = out;
+            if (lslot == PK_NO_SLOT) {
+                first_miss = min(first_miss, (uint32_t)(e - a));
+                if (res < 0) set_status(status, res);
+            } else if (res < 0) {
+                arg_hit = e > arg_hit ? e : arg_hit;
+            }
+        }
+    }
+    const uint32_t hm = __reduce_min_sync(kFull, first_miss);
+    const int64_t h = hm != 0xffffffffu ? (int64_t)hm : (b > a ? b - a : 0);
+    __syncwarp();
+    for (int64_t x = a + lane; x < a + h; x += 32) {  // below h_r: looked up, not stored
+        result[x] = PK_STORE_SKIPPED;
+        slot_out[x] = PK_NO_SLOT;
+    }
+    if (r < R && lane == 0) hit[r] = (int32_t)h;
+    if (arg_hit >= a + h) set_status(status, PK_ERR_ARG);
+    count_claims(&block_claims, claims, counter);
+}
+
+// Few long requests: one warp per 32 consecutive keys; k_lookup_store_tail
+// then finds h_r and relabels.
+__global__ void __launch_bounds__(256)
+k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity, unsigned long long *counter,
+               unsigned long long epoch, const uint8_t *__restrict__ keys, const uint32_t *__restrict__ new_slots,
+               const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capacity, uint32_t *__restrict__ slots,
+               int32_t *__restrict__ result, uint32_t *__restrict__ slot_out, int32_t *status) {
+    __shared__ unsigned long long block_claims;
+    if (threadIdx.x == 0) block_claims = 0;
+    __syncthreads();
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
+    const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const uint32_t lane = threadIdx.x & 31;
+    const int64_t total = R == 0 ? 0 : __ldg(key_off + R);
+    const int64_t end = total < (int64_t)key_capacity ? total : (int64_t)key_capacity;
+    unsigned long long cnt = 0;
+    if (lane == 0) cnt = ld_volatile_u64(counter);
+    const bool fast = __shfl_sync(kFull, cnt, 0) + key_capacity < capacity;
+    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast};
+    int32_t res = PK_STORE_SKIPPED;
+    uint32_t out = PK_NO_SLOT, lslot = PK_NO_SLOT;
+    ProbeKey s;
+    s.pending = false;
+    if (e < end) {
+        const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
+        if (is_zero(key))
+            res = PK_ERR_RESERVED_KEY;  // the empty marker: never stored, so a miss
+        else
+            probe_start(s, key, (uint64_t)e, mask, __ldg(new_slots + e) != PK_NO_SLOT);
+    }
+    uint32_t claims = 0;
+    warp_claim<true>(c, s, res, out, lslot, claims);
+    if (e < end) {
+        slots[e] = lslot;
+        result[e] = res;
+        slot_out[e] = out;
+        if (lslot == PK_NO_SLOT && res < 0) set_status(status, res);
+    }
+    count_claims(&block_claims, claims, counter);
+}
+
+// One warp per request: h_r = the first miss (slot PK_NO_SLOT), entries below
+// it relabelled PK_STORE_SKIPPED, and PK_ERR_ARG reported for a hit at or
+// after h_r whose slot was PK_NO_SLOT.
+__global__ void __launch_bounds__(256)
+k_lookup_store_tail(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capacity,
+                    const uint32_t *__restrict__ slots, int32_t *__restrict__ hit, int32_t *__restrict__ result,
+                    uint32_t *__restrict__ slot_out, int32_t *status) {
+    pk::pdl_launch_dependents();
+    pk::pdl_wait();
+    const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const uint32_t lane = threadIdx.x & 31;
+    if (r >= R) return;
+    const int64_t a = __ldg(key_off + r);
+    int64_t b = __ldg(key_off + r + 1);
+    if ((uint64_t)b > key_capacity) b = (int64_t)key_capacity;
+    int64_t h = b > a ? b - a : 0;
+    bool arg = false;
+    for (int64_t base = a; base < b; base += 32) {
+        const int64_t x = base + lane;
+        const bool in = x < b;
+        const uint32_t sl = in ? slots[x] : 0u;
+        const uint32_t ball = __ballot_sync(kFull, in && sl == PK_NO_SLOT);
+        const int64_t hb = ball ? base - a + (__ffs(ball) - 1) : INT64_MAX;
+        if (h == b - a && hb < h) h = hb;  // first miss found in this group
+        if (in && x >= a + h) arg |= sl != PK_NO_SLOT && result[x] == PK_ERR_ARG;
+    }
+    for (int64_t x = a + lane; x < a + h; x += 32) {
+        result[x] = PK_STORE_SKIPPED;
+        slot_out[x] = PK_NO_SLOT;
+    }
+    if (lane == 0) hit[r] = (int32_t)h;
+    if (arg) set_status(status, PK_ERR_ARG);
 }
 
 // Store, kernel 2 of 2: the lowest claimant of each new key writes its slot.
@@ -797,8 +1009,8 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
         const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
         if (claimable(key, slots[e], res)) probe_start(s, key, e, mask);
     }
-    uint32_t claims = 0;
-    warp_claim(c, s, res, out, claims);
+    uint32_t claims = 0, lslot;
+    warp_claim<false>(c, s, res, out, lslot, claims);
     if (e < n) {
         result[e] = res;
         if (res == PK_STORE_PENDING) {
@@ -881,6 +1093,33 @@ cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const u
     }
     if (e == cudaSuccess)
         e = pk_launch(k_store_finalize, grid_for(n, 256), 256, s, ctx->table, slots, n, key_off, R, result, slot_out);
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+cudaError_t pk_launch_lookup_store(const pk_ctx *ctx, unsigned long long epoch, const uint8_t *keys,
+                                   const uint32_t *new_slots, const int64_t *key_off, uint32_t R,
+                                   uint64_t key_capacity, int32_t *hit_chunks, uint32_t *slots, int32_t *result,
+                                   uint32_t *slot_out, int32_t *status, cudaStream_t s) {
+    if (R == 0) return cudaSuccess;
+    const uint64_t mask = ctx->capacity - 1;
+    cudaError_t e;
+    if (per_request(R, key_capacity)) {
+        e = pk_launch(k_lookup_store_req, grid_for(32ull * R, 256), 256, s, ctx->table, mask, ctx->max_probe,
+                      ctx->capacity, ctx->counter_dev, epoch, keys, new_slots, key_off, R, key_capacity, slots,
+                      hit_chunks, result, slot_out, status);
+    } else {
+        e = key_capacity == 0
+                ? cudaSuccess
+                : pk_launch(k_lookup_store, grid_for(key_capacity, 256), 256, s, ctx->table, mask, ctx->max_probe,
+                            ctx->capacity, ctx->counter_dev, epoch, keys, new_slots, key_off, R, key_capacity, slots,
+                            result, slot_out, status);
+        if (e == cudaSuccess)
+            e = pk_launch(k_lookup_store_tail, grid_for(32ull * R, 256), 256, s, key_off, R, key_capacity,
+                          (const uint32_t *)slots, hit_chunks, result, slot_out, status);
+    }
+    if (e == cudaSuccess && key_capacity)
+        e = pk_launch(k_store_finalize, grid_for(key_capacity, 256), 256, s, ctx->table, new_slots, key_capacity,
+                      key_off, R, result, slot_out);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 

@@ -86,6 +86,7 @@ def lib() -> ctypes.CDLL:
                                                   _U64, _VP, _VP]),
             "pk_lookup": (ctypes.c_int, [_VP, _VP, _VP, _U32, _U64, _VP, _VP, _VP, _VP]),
             "pk_store": (ctypes.c_int, [_VP, _VP, _VP, _U64, _VP, _VP, _U32, _VP, _VP, _VP, _VP]),
+            "pk_lookup_store": (ctypes.c_int, [_VP, _VP, _VP, _VP, _U32, _U64, _VP, _VP, _VP, _VP, _VP, _VP]),
             "pk_entries": (ctypes.c_int, [_VP, ctypes.POINTER(ctypes.c_uint64), _VP]),
             "pk_store_noalloc": (ctypes.c_int, [ctypes.POINTER(pk_config), _VP, _VP, _U64, _VP, _VP, _U32, _VP, _VP,
                                                 _VP, _VP]),
@@ -261,6 +262,15 @@ def pk_store(ctx: int, keys: torch.Tensor, slots: torch.Tensor, result: torch.Te
     R = 0 if key_off is None else key_off.numel() - 1
     _check(lib().pk_store(ctx, _p(keys), _p(slots), n, _p(key_off), _p(hit_chunks), R, _p(result), _p(slot_out),
                           _p(status), _s(stream)), "pk_store")
+
+
+def pk_lookup_store(ctx: int, keys: torch.Tensor, new_slots: torch.Tensor, key_off: torch.Tensor,
+                    hit_chunks: torch.Tensor, slots: torch.Tensor, result: torch.Tensor, slot_out: torch.Tensor,
+                    status: torch.Tensor, stream=None) -> None:
+    R = key_off.numel() - 1
+    _check(lib().pk_lookup_store(ctx, _p(keys), _p(new_slots), _p(key_off), R, keys.numel() // 32,
+                                 _p(hit_chunks), _p(slots), _p(result), _p(slot_out), _p(status), _s(stream)),
+           "pk_lookup_store")
 
 
 def pk_table_save(ctx: int, dst: torch.Tensor, stream=None) -> None:

@@ -144,6 +144,21 @@ class KeyTable:
         pk.pk_store(self.ctx, keys, slots, result, slot_out, self.status, key_off, hit, self.stream)
         return result, slot_out
 
+    def lookup_store(self, keys, key_off, new_slots):
+        """lookup followed by store of the miss ranges, in one pass: returns
+        (hit, slots, result, slot_out) as the two calls would."""
+        R = key_off.numel() - 1
+        n = keys.shape[0]
+        new_slots = _dev(new_slots if isinstance(new_slots, torch.Tensor) else np.asarray(new_slots, np.uint32),
+                         torch.int32, self.device)
+        hit = torch.empty(R, dtype=torch.int32, device=self.device)
+        slots = torch.empty(n, dtype=torch.int32, device=self.device)
+        result = torch.empty(n, dtype=torch.int32, device=self.device)
+        slot_out = torch.empty(n, dtype=torch.int32, device=self.device)
+        pk.pk_lookup_store(self.ctx, keys, new_slots, key_off, hit, slots, result, slot_out, self.status,
+                           self.stream)
+        return hit, slots, result, slot_out
+
     def seed(self, seed_keys, filler, target_entries: int) -> int:
         """Pre-fill: seed keys in order (slot = list index), then filler keys
         (continuing the index) until the table holds target_entries entries."""

@@ -123,5 +123,6 @@ def test_null_context_rejected(pk):
     L = pk.lib()
     assert L.pk_lookup(None, None, None, 0, 0, None, None, None, None) == pk.PK_ERR_ARG
     assert L.pk_store(None, None, None, 0, None, None, 0, None, None, None, None) == pk.PK_ERR_ARG
+    assert L.pk_lookup_store(None, None, None, None, 0, 0, None, None, None, None, None, None) == pk.PK_ERR_ARG
     assert L.pk_derive_keys(None, None, 0, None, 0, None, None, 0, None, None, 0, None, None) == pk.PK_ERR_ARG
     assert L.pk_destroy(None) == pk.PK_ERR_ARG
