@@ -13,11 +13,13 @@
 //   epoch    number of the store call that inserted the key (0 while empty)
 struct alignas(32) pk_entry {
     uint32_t k[4];
-    uint32_t slot;
-    uint32_t owner;
+    uint32_t slot;   // slot and owner form one little-endian 64-bit word
+    uint32_t owner;  // (owner in the high half), raised by atomicMax
     unsigned long long epoch;
 };
 static_assert(sizeof(pk_entry) == PK_ENTRY_BYTES, "entry layout");
+static_assert(offsetof(pk_entry, owner) == offsetof(pk_entry, slot) + 4 && offsetof(pk_entry, slot) % 8 == 0,
+              "slot and owner form one 64-bit word");
 
 struct pk_ctx {
     uint32_t chunk_tokens;

@@ -11,9 +11,11 @@
 //
 // Lookup (Sec. 2.1: on a local miss the connector queries the store) reads
 // the table only.  Store ("a miss computes and writes new state") inserts
-// missing keys with a 128-bit compare-and-swap on the key, and resolves
-// duplicates within one call to the lowest entry index in a second kernel, so
-// that the result equals processing the entries one at a time in order.
+// missing keys with a 128-bit compare-and-swap on the key; every entry of the
+// call holding a new key bids for it with a 64-bit atomicMax on the entry's
+// slot/owner word, so that the lowest entry index's slot is bound, and a
+// second kernel reports each entry's outcome: the result equals processing
+// the entries one at a time in order.
 #include <cuda_runtime.h>
 
 #include "pk_device.cuh"
@@ -134,14 +136,16 @@ struct ProbeKey {
     uint64_t e;       // entry index of the key in the caller's arrays
     uint64_t pos;     // next table position of its probe sequence
     uint32_t probed;  // entries of the sequence examined so far
+    uint32_t slot;    // store: the slot to bind if the key is inserted
     bool pending;     // not decided yet
     bool may_claim;   // lookup-and-store: the key may be inserted (its slot is valid)
 };
 
 __device__ __forceinline__ void probe_start(ProbeKey &s, const uint4 &key, uint64_t e, uint64_t mask,
-                                            bool may_claim = true) {
+                                            uint32_t slot = 0, bool may_claim = true) {
     s.key = key;
     s.e = e;
+    s.slot = slot;
     s.pos = home_of(key) & mask;
     s.probed = 0;
     s.pending = true;
@@ -347,9 +351,9 @@ k_first_miss(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capac
 // Store, kernel 1 of 2: find or claim each key's entry.
 //   pre-existing key (epoch of an earlier call): PRESENT with its slot, final
 //   key absent: CAS the key into the first empty entry
-//   key claimed in this call (by anyone): record the lowest claimant index in
-//   `owner` (atomicMax of ~index) and leave PENDING with the entry position
-//   in slot_out for kernel 2.
+//   key claimed in this call (by anyone): bid (~index, slot) on the entry's
+//   slot/owner word and leave PENDING with the entry position in slot_out
+//   for kernel 2.
 // Capacity: when the table holds few enough entries that this call cannot
 // fill it (count + n < capacity), claims are counted once per block at the
 // end.  Otherwise a new key is refused (TABLE_FULL) once the count reaches
@@ -359,16 +363,23 @@ k_first_miss(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capac
 // ---------------------------------------------------------------------------
 enum Examine { kAdvance, kDone, kClaimedHere };
 
+// Bid of entry index e (me = ~e) with its slot for a key new in this call:
+// the entry's slot/owner word ends at the maximum bid, that of the lowest
+// index, carrying that index's slot.
+__device__ __forceinline__ void bid(pk_entry *ent, uint32_t me, uint32_t my_slot) {
+    atomicMax(reinterpret_cast<unsigned long long *>(&ent->slot), ((unsigned long long)me << 32) | my_slot);
+}
+
 // Examine entry `ent` (position pos) whose key was read as `cur`.
-// kFused (lookup-and-store): `present` tells whether the key was in the
-// table when the call started (inserted by an earlier call: epoch set and
-// not this call's), with its slot in lslot; a key that may not be inserted
+// kFused (lookup-and-store): `lslot` receives the slot of a key that was in
+// the table when the call started (inserted by an earlier call: epoch set
+// and not this call's), else PK_NO_SLOT; a key that may not be inserted
 // (!may_claim) ends with PK_ERR_ARG and leaves the table untouched.
 template <bool kFused>
 __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cur, const uint4 &key, uint32_t me,
-                                           unsigned long long epoch, bool fast, unsigned long long *counter,
-                                           uint64_t capacity, bool may_claim, int32_t &res, uint32_t &out,
-                                           uint32_t &lslot) {
+                                           uint32_t my_slot, unsigned long long epoch, bool fast,
+                                           unsigned long long *counter, uint64_t capacity, bool may_claim,
+                                           int32_t &res, uint32_t &out, uint32_t &lslot) {
     uint4 *kp = reinterpret_cast<uint4 *>(ent->k);
     lslot = PK_NO_SLOT;
 #pragma unroll 1
@@ -381,14 +392,15 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
             (cur.z == 0 || cur.z == key.z) && (cur.w == 0 || cur.w == key.w))
             cur = atomicCAS(kp, key, key);
         if (same(cur, key)) {
-            const unsigned long long ep = ld_volatile_u64(&ent->epoch);
+            const uint4 m = ld_volatile_v4(&ent->slot);  // slot, owner, epoch in one read
+            const unsigned long long ep = ((unsigned long long)m.w << 32) | m.z;
             if (ep != 0ull && ep != epoch) {  // inserted by an earlier call
-                const uint32_t sl = *(volatile uint32_t *)&ent->slot;
+                const uint32_t sl = m.x;
                 if (kFused) lslot = sl;
                 res = (!kFused || may_claim) ? PK_STORE_PRESENT : PK_ERR_ARG;
                 out = (!kFused || may_claim) ? sl : PK_NO_SLOT;
             } else if (!kFused || may_claim) {  // claimed during this call
-                atomicMax(&ent->owner, me);
+                bid(ent, me, my_slot);
                 res = PK_STORE_PENDING;
                 out = (uint32_t)pos;
             } else {
@@ -413,7 +425,7 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
         const uint4 old = atomicCAS(kp, make_uint4(0, 0, 0, 0), key);
         if (is_zero(old)) {  // claimed
             *(volatile unsigned long long *)&ent->epoch = epoch;
-            atomicMax(&ent->owner, me);
+            bid(ent, me, my_slot);
             res = PK_STORE_PENDING;
             out = (uint32_t)pos;
             if (fast) return kClaimedHere;  // counted once per block at the end
@@ -461,6 +473,7 @@ __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, Probe
     const uint32_t wprobed = full ? s.probed : __shfl_sync(kFull, s.probed, rd.owner);
     const uint64_t we = full ? s.e : __shfl_sync(kFull, s.e, rd.owner);
     const bool wmay = !kFused || (full ? s.may_claim : __shfl_sync(kFull, (int)s.may_claim, rd.owner) != 0);
+    const uint32_t wslot = full ? s.slot : __shfl_sync(kFull, s.slot, rd.owner);
     const uint64_t base0 = wpos & ~(uint64_t)(win - 1);
     const uint32_t j0 = (uint32_t)(wpos - base0);
     const uint64_t wb = (base0 + (uint64_t)rd.j * win) & c.mask;
@@ -495,8 +508,8 @@ __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, Probe
     uint32_t dprobed = 0;
     if (decider) {
         const uint64_t epos = wb + (uint32_t)cand;
-        const Examine x = examine<kFused>(c.table + epos, epos, cv, k, ~(uint32_t)we, c.epoch, c.fast, c.counter,
-                                          c.capacity, wmay, dres, dout, dls);
+        const Examine x = examine<kFused>(c.table + epos, epos, cv, k, ~(uint32_t)we, wslot, c.epoch, c.fast,
+                                          c.counter, c.capacity, wmay, dres, dout, dls);
         if (x == kClaimedHere) ++claims;
         if (x == kAdvance) {  // lost the entry to a different key: continue after it
             dadv = true;
@@ -622,7 +635,8 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
     s.pending = false;
     if (active) {
         const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
-        if (claimable(key, slots[e], res)) probe_start(s, key, e, mask);
+        const uint32_t sl = slots[e];
+        if (claimable(key, sl, res)) probe_start(s, key, e, mask, sl);
     }
     uint32_t claims = 0, lslot;
     warp_claim<false>(c, s, res, out, lslot, claims);
@@ -689,7 +703,7 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
                 const int64_t e = cursor + rank;
                 int32_t res;
                 if (claimable(kin, sin, res)) {
-                    probe_start(s, kin, (uint64_t)e, mask);
+                    probe_start(s, kin, (uint64_t)e, mask, sin);
                 } else {
                     result[e] = res;
                     slot_out[e] = PK_NO_SLOT;
@@ -784,7 +798,7 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
                     set_status(status, PK_ERR_RESERVED_KEY);
                     first_miss = min(first_miss, (uint32_t)(e - a));
                 } else {
-                    probe_start(s, kin, (uint64_t)e, mask, sin != PK_NO_SLOT);
+                    probe_start(s, kin, (uint64_t)e, mask, sin, sin != PK_NO_SLOT);
                 }
             }
             const uint32_t nF = __popc(F);
@@ -854,10 +868,11 @@ k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capa
     s.pending = false;
     if (e < end) {
         const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
+        const uint32_t sl = __ldg(new_slots + e);
         if (is_zero(key))
             res = PK_ERR_RESERVED_KEY;  // the empty marker: never stored, so a miss
         else
-            probe_start(s, key, (uint64_t)e, mask, __ldg(new_slots + e) != PK_NO_SLOT);
+            probe_start(s, key, (uint64_t)e, mask, sl, sl != PK_NO_SLOT);
     }
     uint32_t claims = 0;
     warp_claim<true>(c, s, res, out, lslot, claims);
@@ -904,12 +919,13 @@ k_lookup_store_tail(const int64_t *__restrict__ key_off, uint32_t R, uint64_t ke
     if (arg) set_status(status, PK_ERR_ARG);
 }
 
-// Store, kernel 2 of 2: the lowest claimant of each new key writes its slot.
-// In range mode, entries past key_off[R] (not keys of this batch) are skipped.
+// Store, kernel 2 of 2: each PENDING entry reads its key's slot/owner word,
+// final once every claim is in: the lowest claimant is INSERTED, the others
+// PRESENT with its slot.  In range mode, entries past key_off[R] (not keys
+// of this batch) are skipped.
 __global__ void __launch_bounds__(256)
-k_store_finalize(pk_entry *table, const uint32_t *__restrict__ slots, uint64_t n,
-                 const int64_t *__restrict__ key_off, uint32_t R, int32_t *__restrict__ result,
-                 uint32_t *__restrict__ slot_out) {
+k_store_finalize(const pk_entry *table, uint64_t n, const int64_t *__restrict__ key_off, uint32_t R,
+                 int32_t *__restrict__ result, uint32_t *__restrict__ slot_out) {
     pk::pdl_launch_dependents();
     pk::pdl_wait();
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -920,16 +936,9 @@ k_store_finalize(pk_entry *table, const uint32_t *__restrict__ slots, uint64_t n
         return;
     }
     if (result[e] != PK_STORE_PENDING) return;
-    pk_entry *ent = table + slot_out[e];
-    const uint32_t winner = ~ent->owner;
-    if (winner == (uint32_t)e) {
-        ent->slot = slots[e];
-        result[e] = PK_STORE_INSERTED;
-        slot_out[e] = slots[e];
-    } else {
-        result[e] = PK_STORE_PRESENT;
-        slot_out[e] = slots[winner];
-    }
+    const unsigned long long w = *reinterpret_cast<const unsigned long long *>(&table[slot_out[e]].slot);
+    result[e] = ~(uint32_t)(w >> 32) == (uint32_t)e ? PK_STORE_INSERTED : PK_STORE_PRESENT;
+    slot_out[e] = (uint32_t)w;
 }
 
 // After a table load: every stored entry counts as inserted before any later
@@ -1007,7 +1016,8 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
     s.pending = false;
     if (active) {
         const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
-        if (claimable(key, slots[e], res)) probe_start(s, key, e, mask);
+        const uint32_t sl = slots[e];
+        if (claimable(key, sl, res)) probe_start(s, key, e, mask, sl);
     }
     uint32_t claims = 0, lslot;
     warp_claim<false>(c, s, res, out, lslot, claims);
@@ -1025,20 +1035,13 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
 }
 
 __global__ void __launch_bounds__(256)
-k_noalloc_finalize(pk_entry *table, const NoallocScratch *sc, const uint32_t *__restrict__ slots, uint64_t n,
-                   int32_t *__restrict__ result, uint32_t *__restrict__ slot_out) {
+k_noalloc_finalize(const pk_entry *table, const NoallocScratch *sc, uint64_t n, int32_t *__restrict__ result,
+                   uint32_t *__restrict__ slot_out) {
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (e >= n || result[e] != PK_STORE_PENDING) return;
-    pk_entry *ent = table + sc->pos[e];
-    const uint32_t winner = ~ent->owner;
-    if (winner == (uint32_t)e) {
-        ent->slot = slots[e];
-        result[e] = PK_STORE_INSERTED;
-        slot_out[e] = slots[e];
-    } else {
-        result[e] = PK_STORE_PRESENT;
-        slot_out[e] = slots[winner];
-    }
+    const unsigned long long w = *reinterpret_cast<const unsigned long long *>(&table[sc->pos[e]].slot);
+    result[e] = ~(uint32_t)(w >> 32) == (uint32_t)e ? PK_STORE_INSERTED : PK_STORE_PRESENT;
+    slot_out[e] = (uint32_t)w;
 }
 
 unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1) / block); }
@@ -1092,7 +1095,8 @@ cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const u
                       ctx->counter_dev, epoch, keys, slots, n, key_off, hit_chunks, R, result, slot_out, status);
     }
     if (e == cudaSuccess)
-        e = pk_launch(k_store_finalize, grid_for(n, 256), 256, s, ctx->table, slots, n, key_off, R, result, slot_out);
+        e = pk_launch(k_store_finalize, grid_for(n, 256), 256, s, (const pk_entry *)ctx->table, n, key_off, R, result,
+                      slot_out);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -1118,8 +1122,8 @@ cudaError_t pk_launch_lookup_store(const pk_ctx *ctx, unsigned long long epoch, 
                           (const uint32_t *)slots, hit_chunks, result, slot_out, status);
     }
     if (e == cudaSuccess && key_capacity)
-        e = pk_launch(k_store_finalize, grid_for(key_capacity, 256), 256, s, ctx->table, new_slots, key_capacity,
-                      key_off, R, result, slot_out);
+        e = pk_launch(k_store_finalize, grid_for(key_capacity, 256), 256, s, (const pk_entry *)ctx->table,
+                      key_capacity, key_off, R, result, slot_out);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -1156,6 +1160,6 @@ cudaError_t pk_launch_store_noalloc(pk_entry *table, uint32_t capacity_log2, uin
     k_noalloc_scan<<<(unsigned)(scan_blocks < 152 * 8 ? scan_blocks : 152 * 8), 256, 0, s>>>(table, capacity, sc);
     k_noalloc_claim<<<grid_for(n, 256), 256, 0, s>>>(table, capacity - 1, max_probe, capacity, sc, keys, slots, n,
                                                       key_off, hit_chunks, key_off ? R : 0, result, slot_out, status);
-    k_noalloc_finalize<<<grid_for(n, 256), 256, 0, s>>>(table, sc, slots, n, result, slot_out);
+    k_noalloc_finalize<<<grid_for(n, 256), 256, 0, s>>>(table, sc, n, result, slot_out);
     return cudaGetLastError();
 }
