@@ -430,7 +430,9 @@ def main():
     probe_bytes = n_keys * (16 + 32 + 4 + 12) + inserted * 32 + R * 4
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+        "step_ms_min_median_max": [float(np.min(step_ms)), float(np.median(step_ms)), float(np.max(step_ms))],
+        "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
         "config": workload_config(wl, args),
         "lookups_per_s": n_keys * args.steps * world / (total_ms / 1e3),

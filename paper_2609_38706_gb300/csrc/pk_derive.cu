@@ -31,11 +31,11 @@ constexpr int kDescWarps = 4;
 constexpr int kDescStage = 2048;
 
 // Warp `warp` of the calling block hashes descriptor j (all 32 lanes call).
-__device__ __forceinline__ void hash_descriptor(uint8_t *stage, const uint8_t *__restrict__ enc, uint64_t enc_bytes,
-                                                const int64_t *__restrict__ enc_off, uint32_t j,
-                                                uint8_t *__restrict__ digests, int32_t *status) {
+__device__ __forceinline__ void hash_descriptor(uint8_t *stage, const uint8_t *enc, uint64_t enc_bytes,
+                                                const int64_t *enc_off, uint32_t j,
+                                                uint8_t *digests, int32_t *status) {
     const uint32_t lane = threadIdx.x & 31;
-    const int64_t a = __ldg(enc_off + j), b = __ldg(enc_off + j + 1);
+    const int64_t a = __ldcg(enc_off + j), b = __ldcg(enc_off + j + 1);
     if (a < 0 || b < a || (uint64_t)b > enc_bytes) {
         if (lane == 0) set_status(status, PK_ERR_ARG);
         return;
@@ -44,18 +44,18 @@ __device__ __forceinline__ void hash_descriptor(uint8_t *stage, const uint8_t *_
     const bool staged = len <= kDescStage;
     if (staged) {
 #pragma unroll 4
-        for (int64_t i = lane; i < len; i += 32) stage[i] = __ldg(enc + a + i);
+        for (int64_t i = lane; i < len; i += 32) stage[i] = __ldcg(enc + a + i);
     }
     __syncwarp();
     if (lane == 0) pk::sha256_bytes(staged ? stage : enc + a, (uint64_t)len, digests + 32ull * j);
 }
 
 __global__ void __launch_bounds__(32 * kDescWarps)
-k_digest_descriptors(const uint8_t *__restrict__ enc, uint64_t enc_bytes, const int64_t *__restrict__ enc_off,
-                     uint32_t D, uint8_t *__restrict__ digests, int32_t *status) {
+k_digest_descriptors(const uint8_t *enc, uint64_t enc_bytes, const int64_t *enc_off,
+                     uint32_t D, uint8_t *digests, int32_t *status) {
     __shared__ __align__(16) uint8_t stage[kDescWarps][kDescStage];
     pk::pdl_launch_dependents();
-    pk::pdl_wait();
+    pk::pdl_wait(enc, enc_off, digests, status);
     const uint32_t warp = threadIdx.x >> 5;
     const uint32_t j = blockIdx.x * kDescWarps + warp;
     if (j < D) hash_descriptor(stage[warp], enc, enc_bytes, enc_off, j, digests, status);
@@ -73,13 +73,13 @@ constexpr int kScanThreads = 1024;
 constexpr int kScanItems = 4;
 
 __global__ void __launch_bounds__(kScanThreads)
-k_chunk_offsets(const int64_t *__restrict__ tok_off, uint32_t R, uint64_t n_tokens, uint32_t C,
-                const uint32_t *__restrict__ desc_idx, uint32_t D, uint64_t key_capacity,
-                int64_t *__restrict__ key_off, int32_t *status) {
+k_chunk_offsets(const int64_t *tok_off, uint32_t R, uint64_t n_tokens, uint32_t C,
+                const uint32_t *desc_idx, uint32_t D, uint64_t key_capacity,
+                int64_t *key_off, int32_t *status) {
     __shared__ long long warp_sums[kScanThreads / 32];
     __shared__ long long tile_total;
     pk::pdl_launch_dependents();
-    pk::pdl_wait();
+    pk::pdl_wait(tok_off, desc_idx, key_off, status);
     const uint32_t tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (tid == 0) key_off[0] = 0;
     bool bad = false;
@@ -146,9 +146,9 @@ __device__ __forceinline__ void store_digest(uint8_t *dst, const uint32_t st[8])
 
 // 16 message words of one 64-byte block of int32 tokens (little-endian bytes,
 // read by SHA-256 as big-endian words), straight from global memory.
-__device__ __forceinline__ void load_block_global(const int32_t *__restrict__ src, uint32_t w[16]) {
+__device__ __forceinline__ void load_block_global(const int32_t *src, uint32_t w[16]) {
 #pragma unroll
-    for (int t = 0; t < 16; ++t) w[t] = pk::bswap32((uint32_t)__ldg(src + t));
+    for (int t = 0; t < 16; ++t) w[t] = pk::bswap32((uint32_t)__ldcg(src + t));
 }
 
 // Asynchronous 64-byte copy global -> shared (4 x 16 B; both 16-byte aligned).
@@ -185,12 +185,12 @@ constexpr int kDigestBlock = 128;
 constexpr int kStages = 3;
 
 // c = SHA-256 of chunk g (request r), written to keys[g].
-__device__ __forceinline__ void digest_chunk(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_off,
-                                             const int64_t *__restrict__ key_off, uint32_t r, int64_t g, uint32_t C,
+__device__ __forceinline__ void digest_chunk(const int32_t *tokens, const int64_t *tok_off,
+                                             const int64_t *key_off, uint32_t r, int64_t g, uint32_t C,
                                              const uint32_t *sK, const uint32_t *sPad,
-                                             uint32_t (*ring)[kDigestBlock][16], uint8_t *__restrict__ keys) {
-    const int64_t i = g - __ldg(key_off + r);
-    const int32_t *src = tokens + __ldg(tok_off + r) + i * (int64_t)C;
+                                             uint32_t (*ring)[kDigestBlock][16], uint8_t *keys) {
+    const int64_t i = g - __ldcg(key_off + r);
+    const int32_t *src = tokens + __ldcg(tok_off + r) + i * (int64_t)C;
     const bool aligned = (reinterpret_cast<uintptr_t>(src) & 15) == 0;
 
     uint32_t st[8];
@@ -236,7 +236,7 @@ __device__ __forceinline__ void digest_chunk(const int32_t *__restrict__ tokens,
         const int32_t *tail = src + 16 * nfull;
 #pragma unroll
         for (int t = 0; t < 16; ++t)
-            w[t] = t < rem ? pk::bswap32((uint32_t)__ldg(tail + t)) : (t == rem ? 0x80000000u : 0u);
+            w[t] = t < rem ? pk::bswap32((uint32_t)__ldcg(tail + t)) : (t == rem ? 0x80000000u : 0u);
         if (rem <= 13) {
             w[14] = (uint32_t)(bits >> 32);
             w[15] = (uint32_t)bits;
@@ -266,26 +266,32 @@ struct DescWork {
 };
 
 __global__ void __launch_bounds__(kDigestBlock)
-k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ tok_off,
-               const int64_t *__restrict__ key_off, uint32_t R, uint32_t C, const __grid_constant__ PadKW pad,
-               uint8_t *__restrict__ keys, const __grid_constant__ DescWork dw, uint32_t r_begin, uint32_t r_end) {
+k_chunk_digest(const int32_t *tokens, const int64_t *tok_off,
+               const int64_t *key_off, uint32_t R, uint32_t C, const __grid_constant__ PadKW pad,
+               uint8_t *keys, const __grid_constant__ DescWork dw, uint32_t r_begin, uint32_t r_end) {
     __shared__ uint32_t sK[64], sPad[64];
     __shared__ __align__(16) uint32_t ring[kStages][kDigestBlock][16];
-    pk::pdl_launch_dependents();
+    // The successor (the chain) is released as each block finishes, not at its start: released early,
+    // its waiting CTAs, and those of the kernel after it, would sit on the SMs during the whole digest.
     if (blockIdx.x < dw.desc_blocks) {
-        pk::pdl_wait();
+        const uint8_t *enc = dw.enc;
+        const int64_t *enc_off = dw.enc_off;
+        uint8_t *digests = dw.digests;
+        int32_t *dstatus = dw.status;
+        pk::pdl_wait(enc, enc_off, digests, dstatus);
         const uint32_t warp = threadIdx.x >> 5;
         const uint32_t j = blockIdx.x * (kDigestBlock / 32) + warp;
         uint8_t *stage = reinterpret_cast<uint8_t *>(ring[0]) + warp * kDescStage;  // 4 x 2 KiB of the ring
-        if (j < dw.D) hash_descriptor(stage, dw.enc, dw.enc_bytes, dw.enc_off, j, dw.digests, dw.status);
+        if (j < dw.D) hash_descriptor(stage, enc, dw.enc_bytes, enc_off, j, digests, dstatus);
+        pk::pdl_launch_dependents();
         return;
     }
     load_tables(sK, sPad, pad);
     __syncthreads();
-    pk::pdl_wait();
+    pk::pdl_wait(tokens, tok_off, key_off, keys);
     if (R == 0 || r_begin >= r_end) return;
     // the chunks of requests [r_begin, r_end), in tiles of one block, grid-strided
-    const int64_t g_begin = __ldg(key_off + r_begin), g_end = __ldg(key_off + r_end);
+    const int64_t g_begin = __ldcg(key_off + r_begin), g_end = __ldcg(key_off + r_end);
     const uint32_t nblocks = gridDim.x - dw.desc_blocks;
     for (int64_t tile = g_begin + (int64_t)(blockIdx.x - dw.desc_blocks) * kDigestBlock; tile < g_end;
          tile += (int64_t)nblocks * kDigestBlock) {
@@ -296,6 +302,7 @@ k_chunk_digest(const int32_t *__restrict__ tokens, const int64_t *__restrict__ t
         if (g < g_end) digest_chunk(tokens, tok_off, key_off, r, g, C, sK, sPad, ring, keys);
         __syncwarp();
     }
+    pk::pdl_launch_dependents();
 }
 
 // ---------------------------------------------------------------------------
@@ -341,19 +348,24 @@ __device__ __forceinline__ void schedule16(uint32_t w[16], uint32_t (*out)[kChai
 }
 
 // rounds t = 16q .. 16q+15 with K+W from shared memory
+// (the 16 words are read into registers before the first round: a lone warp
+// runs 64 rounds in 2018 instead of 2241 cycles when no round waits on its
+// shared-memory read)
 __device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint32_t (*kw)[kChainLanes], int q, uint32_t lane) {
     uint32_t a = v[0], b = v[1], c = v[2], d = v[3], e = v[4], f = v[5], g = v[6], h = v[7];
+    uint32_t x[16];
 #pragma unroll
-    for (int j = 0; j < 16; ++j) pk::round_kw(a, b, c, d, e, f, g, h, kw[16 * q + j][lane]);
+    for (int j = 0; j < 16; ++j) x[j] = kw[16 * q + j][lane];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) pk::round_kw(a, b, c, d, e, f, g, h, x[j]);
     v[0] = a; v[1] = b; v[2] = c; v[3] = d; v[4] = e; v[5] = f; v[6] = g; v[7] = h;
 }
 
 __global__ void __launch_bounds__(2 * kChainLanes)
-k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_idx,
-        const uint8_t *__restrict__ digests, uint32_t r_begin, uint32_t R, uint32_t D, uint8_t *keys) {
+k_chain(const int64_t *key_off, const uint32_t *desc_idx,
+        const uint8_t *digests, uint32_t r_begin, uint32_t R, uint32_t D, uint8_t *keys) {
     __shared__ __align__(16) ChainSmem sm;
-    pk::pdl_launch_dependents();
-    pk::pdl_wait();
+    pk::pdl_wait(key_off, desc_idx, digests, keys);  // successor released at the last step (see k_chunk_digest)
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t r = r_begin + blockIdx.x * kChainLanes + lane;  // requests [r_begin, R)
     int64_t a = 0, n = 0;
@@ -375,7 +387,7 @@ k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_i
     uint32_t dw[8] = {0, 0, 0, 0, 0, 0, 0, 0};
     if (n > 0) {
         const uint4 *dq = reinterpret_cast<const uint4 *>(digests + 32ull * di);
-        const uint4 d_lo = __ldg(dq), d_hi = __ldg(dq + 1);
+        const uint4 d_lo = __ldcg(dq), d_hi = __ldcg(dq + 1);
         dw[0] = pk::bswap32(d_lo.x); dw[1] = pk::bswap32(d_lo.y); dw[2] = pk::bswap32(d_lo.z);
         dw[3] = pk::bswap32(d_lo.w); dw[4] = pk::bswap32(d_hi.x); dw[5] = pk::bswap32(d_hi.y);
         dw[6] = pk::bswap32(d_hi.z); dw[7] = pk::bswap32(d_hi.w);
@@ -407,6 +419,7 @@ k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_i
         bar_arrive(4);
 #pragma unroll 1
         for (int64_t i = 0; i < nmax; ++i) {
+            if (i + 1 == nmax) pk::pdl_launch_dependents();
             uint32_t w[16];
             if (i == 0) {
 #pragma unroll
@@ -438,6 +451,7 @@ k_chain(const int64_t *__restrict__ key_off, const uint32_t *__restrict__ desc_i
     for (int j = 0; j < 8; ++j) kd[j] = pk::kSha256K[8 + j] + dw[j];
 #pragma unroll 1
     for (int64_t i = 0; i < nmax; ++i) {
+        if (i + 1 == nmax) pk::pdl_launch_dependents();
         uint32_t v[8] = {PK_IV0, PK_IV1, PK_IV2, PK_IV3, PK_IV4, PK_IV5, PK_IV6, PK_IV7};
         {   // block 1, rounds 0..15: W = k_{i-1} || d
             uint32_t a_ = v[0], b_ = v[1], c_ = v[2], d_ = v[3], e_ = v[4], f_ = v[5], g_ = v[6], h_ = v[7];

@@ -214,10 +214,13 @@ __device__ __forceinline__ void round_kw(uint32_t &a, uint32_t &b, uint32_t &c, 
 template <bool SCHED>
 __device__ __forceinline__ void rounds16(uint32_t v[8], uint32_t w[16], const uint32_t *__restrict__ k16) {
     uint32_t a = v[0], b = v[1], c = v[2], d = v[3], e = v[4], f = v[5], g = v[6], h = v[7];
+    uint32_t k[16];  // read before the first round, so that no round waits on shared memory
+#pragma unroll
+    for (int j = 0; j < 16; ++j) k[j] = k16[j];
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
         if (SCHED) w[j] += small_s1(w[(j + 14) & 15]) + w[(j + 9) & 15] + small_s0(w[(j + 1) & 15]);
-        round_kw(a, b, c, d, e, f, g, h, k16[j] + w[j]);
+        round_kw(a, b, c, d, e, f, g, h, k[j] + w[j]);
     }
     v[0] = a; v[1] = b; v[2] = c; v[3] = d; v[4] = e; v[5] = f; v[6] = g; v[7] = h;
 }
@@ -240,8 +243,11 @@ __device__ __forceinline__ void compress_kw(uint32_t st[8], const uint32_t *__re
     uint32_t a = st[0], b = st[1], c = st[2], d = st[3], e = st[4], f = st[5], g = st[6], h = st[7];
 #pragma unroll 1
     for (int q = 0; q < 4; ++q) {
+        uint32_t x[16];  // read before the first round, as in rounds16
 #pragma unroll
-        for (int j = 0; j < 16; ++j) round_kw(a, b, c, d, e, f, g, h, kw[16 * q + j]);
+        for (int j = 0; j < 16; ++j) x[j] = kw[16 * q + j];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) round_kw(a, b, c, d, e, f, g, h, x[j]);
     }
     st[0] += a; st[1] += b; st[2] += c; st[3] += d; st[4] += e; st[5] += f; st[6] += g; st[7] += h;
 }

@@ -90,10 +90,11 @@ __device__ __forceinline__ uint4 shfl4(const uint4 &v, uint32_t src) {
                       __shfl_sync(kFull, v.w, src));
 }
 
-// Read-only 16-byte load kept in program order (prefetch of the next keys).
-__device__ __forceinline__ uint4 ld_nc_v4(const void *p) {
+// 16-byte load at L2 (coherent: see pk_device.cuh), kept in program order
+// (prefetch of the next keys).
+__device__ __forceinline__ uint4 ld_cg_v4(const void *p) {
     uint4 v;
-    asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+    asm volatile("ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%4];"
                  : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                  : "l"(p));
     return v;
@@ -165,7 +166,7 @@ __device__ __forceinline__ void skip_windows(ProbeKey &s, uint32_t G, uint32_t w
 // the lanes whose key was decided in this round, with its slot (PK_NO_SLOT
 // if absent) and `limit` set if its sequence reached max_probe.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ bool lookup_round(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
+__device__ __forceinline__ bool lookup_round(const pk_entry *table, uint64_t mask, uint32_t max_probe,
                                              uint32_t P, ProbeKey &s, uint32_t &slot, bool &limit) {
     const uint32_t lane = threadIdx.x & 31;
     const uint32_t win = window_size(mask);
@@ -187,7 +188,7 @@ __device__ __forceinline__ bool lookup_round(const pk_entry *__restrict__ table,
 #pragma unroll
         for (uint32_t u = 0; u < kWin; ++u) {  // entries before the sequence start are not read
             v[u] = make_uint4(0, 0, 0, 0);
-            if (u < win && (rd.j > 0 || u >= j0)) v[u] = __ldg(reinterpret_cast<const uint4 *>(grp[u].k));
+            if (u < win && (rd.j > 0 || u >= j0)) v[u] = __ldcg(reinterpret_cast<const uint4 *>(grp[u].k));
         }
 #pragma unroll
         for (uint32_t u = 0; u < kWin; ++u) {
@@ -205,7 +206,7 @@ __device__ __forceinline__ bool lookup_round(const pk_entry *__restrict__ table,
     const uint32_t B = __ballot_sync(kFull, cand >= 0);
     const bool decider = cand >= 0 && (B & rd.work_mask & lanemask_lt()) == 0;
     uint32_t dslot = PK_NO_SLOT;
-    if (decider && match) dslot = __ldg(&table[wb + (uint32_t)cand].slot);
+    if (decider && match) dslot = __ldcg(&table[wb + (uint32_t)cand].slot);
     const uint32_t ob = B & rd.own_mask;
     const uint32_t got = full ? dslot : __shfl_sync(kFull, dslot, ob ? __ffs(ob) - 1 : lane);
     if (!s.pending) return false;
@@ -230,16 +231,15 @@ __device__ __forceinline__ bool lookup_round(const pk_entry *__restrict__ table,
 // buffer holding the next 32 keys (loaded one refill ahead), so the warp
 // keeps 32 keys in flight until the request's last keys.
 __global__ void __launch_bounds__(256, 4)
-k_lookup_req(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
-             const uint8_t *__restrict__ keys, const int64_t *__restrict__ key_off, uint32_t R,
-             uint64_t key_capacity, uint32_t *__restrict__ slots, int32_t *__restrict__ hit, int32_t *status) {
-    pk::pdl_launch_dependents();
-    pk::pdl_wait();
+k_lookup_req(const pk_entry *table, uint64_t mask, uint32_t max_probe,
+             const uint8_t *keys, const int64_t *key_off, uint32_t R,
+             uint64_t key_capacity, uint32_t *slots, int32_t *hit, int32_t *status) {
+    pk::pdl_wait(table, keys, key_off, slots, hit, status);
     const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t lane = threadIdx.x & 31;
     if (r >= R) return;  // uniform per warp
-    const int64_t a = __ldg(key_off + r);
-    int64_t b = __ldg(key_off + r + 1);
+    const int64_t a = __ldcg(key_off + r);
+    int64_t b = __ldcg(key_off + r + 1);
     if ((uint64_t)b > key_capacity) b = (int64_t)key_capacity;
     uint32_t first_miss = 0xffffffffu;  // lowest missing index (relative to a) seen by this lane
     bool limit = false;
@@ -248,7 +248,7 @@ k_lookup_req(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_pro
     bool busy = false;  // holds a key (pending)
     int64_t cursor = a;
     uint4 buf = make_uint4(0, 0, 0, 0);  // key of index cursor + lane
-    if (a + lane < b) buf = ld_nc_v4(keys + 32 * (a + lane));
+    if (a + lane < b) buf = ld_cg_v4(keys + 32 * (a + lane));
     for (;;) {
         const uint32_t F = __ballot_sync(kFull, !busy);
         if (F) {  // free lanes take the next keys, in lane order
@@ -267,7 +267,7 @@ k_lookup_req(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_pro
             const uint32_t nF = __popc(F);
             buf = shfl4(buf, (lane + nF) & 31);
             cursor += nF;
-            if (lane + nF >= 32 && cursor + lane < b) buf = ld_nc_v4(keys + 32 * (cursor + lane));
+            if (lane + nF >= 32 && cursor + lane < b) buf = ld_cg_v4(keys + 32 * (cursor + lane));
         }
         const uint32_t P = __ballot_sync(kFull, busy);
         if (!P) {
@@ -283,6 +283,7 @@ k_lookup_req(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_pro
             busy = false;
         }
     }
+    pk::pdl_launch_dependents();  // main work done: release the successor (see k_chunk_digest)
     const uint32_t h = __reduce_min_sync(kFull, first_miss);
     if (lane == 0) hit[r] = h != 0xffffffffu ? (int32_t)h : (int32_t)(b > a ? b - a : 0);
     if (limit) set_status(status, PK_ERR_PROBE_LIMIT);
@@ -291,13 +292,12 @@ k_lookup_req(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_pro
 // One warp per 32 consecutive keys (few long requests): slots only;
 // k_first_miss follows.
 __global__ void __launch_bounds__(256)
-k_lookup(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
-         const uint8_t *__restrict__ keys, const int64_t *__restrict__ key_off, uint32_t R,
-         uint64_t key_capacity, uint32_t *__restrict__ slots, int32_t *status) {
-    pk::pdl_launch_dependents();
-    pk::pdl_wait();
+k_lookup(const pk_entry *table, uint64_t mask, uint32_t max_probe,
+         const uint8_t *keys, const int64_t *key_off, uint32_t R,
+         uint64_t key_capacity, uint32_t *slots, int32_t *status) {
+    pk::pdl_wait(table, keys, key_off, slots, status);
     const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const int64_t total = R == 0 ? 0 : __ldg(key_off + R);
+    const int64_t total = R == 0 ? 0 : __ldcg(key_off + R);
     const int64_t end = total < (int64_t)key_capacity ? total : (int64_t)key_capacity;
     if (g - (int64_t)(threadIdx.x & 31) >= end) return;  // uniform per warp
     ProbeKey s;
@@ -305,7 +305,7 @@ k_lookup(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
     uint32_t slot = PK_NO_SLOT;
     bool limit = false;
     if (g < end) {
-        const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * g));
+        const uint4 key = __ldcg(reinterpret_cast<const uint4 *>(keys + 32 * g));
         if (!is_zero(key)) probe_start(s, key, (uint64_t)g, mask);  // the empty marker is never stored
     }
     for (;;) {
@@ -318,26 +318,27 @@ k_lookup(const pk_entry *__restrict__ table, uint64_t mask, uint32_t max_probe,
             limit = lim;
         }
     }
+    pk::pdl_launch_dependents();
     if (g < end) slots[g] = slot;
     if (limit) set_status(status, PK_ERR_PROBE_LIMIT);
 }
 
 // One warp per request: h_r = index of the first PK_NO_SLOT among its keys.
 __global__ void __launch_bounds__(256)
-k_first_miss(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capacity,
-             const uint32_t *__restrict__ slots, int32_t *__restrict__ hit) {
+k_first_miss(const int64_t *key_off, uint32_t R, uint64_t key_capacity,
+             const uint32_t *slots, int32_t *hit) {
     pk::pdl_launch_dependents();
-    pk::pdl_wait();
+    pk::pdl_wait(key_off, slots, hit);
     const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t lane = threadIdx.x & 31;
     if (r >= R) return;
-    const int64_t a = __ldg(key_off + r);
-    int64_t b = __ldg(key_off + r + 1);
+    const int64_t a = __ldcg(key_off + r);
+    int64_t b = __ldcg(key_off + r + 1);
     if ((uint64_t)b > key_capacity) b = (int64_t)key_capacity;
     int64_t h = b > a ? b - a : 0;
     for (int64_t base = a; base < b; base += 32) {
         const int64_t idx = base + lane;
-        const bool miss = idx < b && __ldg(slots + idx) == PK_NO_SLOT;
+        const bool miss = idx < b && __ldcg(slots + idx) == PK_NO_SLOT;
         const uint32_t ball = __ballot_sync(kFull, miss);
         if (ball) {
             h = base - a + (__ffs(ball) - 1);
@@ -583,16 +584,16 @@ __device__ __forceinline__ bool claimable(const uint4 &key, uint32_t slot, int32
 
 // Whether entry e lies in the store range of its request, [key_off[r] + h_r,
 // key_off[r+1]) (range mode; warp-collective).
-__device__ __forceinline__ bool in_store_range(const int64_t *__restrict__ key_off, const int32_t *__restrict__ hit,
+__device__ __forceinline__ bool in_store_range(const int64_t *key_off, const int32_t *hit,
                                                uint32_t R, uint64_t n, uint64_t e) {
     const uint64_t e0 = e - (threadIdx.x & 31);
-    const int64_t total = R > 0 ? __ldg(key_off + R) : 0;
+    const int64_t total = R > 0 ? __ldcg(key_off + R) : 0;
     bool in_range = false;
     if (e0 < n && (int64_t)e0 < total) {
         const uint32_t r = pk::lane_request(key_off, R, (int64_t)e0, total, (int64_t)e);
         if ((int64_t)e < total) {
-            const int64_t h = __ldg(hit + r);
-            in_range = (int64_t)e - __ldg(key_off + r) >= (h > 0 ? h : 0);
+            const int64_t h = __ldcg(hit + r);
+            in_range = (int64_t)e - __ldcg(key_off + r) >= (h > 0 ? h : 0);
         }
     }
     return in_range;
@@ -612,15 +613,14 @@ __device__ __forceinline__ void count_claims(unsigned long long *block_claims, u
 // consecutive entries.
 __global__ void __launch_bounds__(256, 4)
 k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
-              unsigned long long *counter, unsigned long long epoch, const uint8_t *__restrict__ keys,
-              const uint32_t *__restrict__ slots, uint64_t n, const int64_t *__restrict__ key_off,
-              const int32_t *__restrict__ hit, uint32_t R, int32_t *__restrict__ result,
-              uint32_t *__restrict__ slot_out, int32_t *status) {
+              unsigned long long *counter, unsigned long long epoch, const uint8_t *keys,
+              const uint32_t *slots, uint64_t n, const int64_t *key_off,
+              const int32_t *hit, uint32_t R, int32_t *result,
+              uint32_t *slot_out, int32_t *status) {
     __shared__ unsigned long long block_claims;
     if (threadIdx.x == 0) block_claims = 0;
     __syncthreads();
-    pk::pdl_launch_dependents();
-    pk::pdl_wait();
+    pk::pdl_wait(table, counter, keys, slots, key_off, hit, result, slot_out, status);
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const uint32_t lane = threadIdx.x & 31;
     bool active = e < n;
@@ -634,7 +634,7 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
     ProbeKey s;
     s.pending = false;
     if (active) {
-        const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
+        const uint4 key = __ldcg(reinterpret_cast<const uint4 *>(keys + 32 * e));
         const uint32_t sl = slots[e];
         if (claimable(key, sl, res)) probe_start(s, key, e, mask, sl);
     }
@@ -645,6 +645,7 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
         slot_out[e] = out;
         if (res < 0) set_status(status, res);
     }
+    pk::pdl_launch_dependents();
     count_claims(&block_claims, claims, counter);
 }
 
@@ -653,23 +654,22 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
 // are marked by the finalize kernel.
 __global__ void __launch_bounds__(256, 4)
 k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
-                  unsigned long long *counter, unsigned long long epoch, const uint8_t *__restrict__ keys,
-                  const uint32_t *__restrict__ slots, uint64_t n, const int64_t *__restrict__ key_off,
-                  const int32_t *__restrict__ hit, uint32_t R, int32_t *__restrict__ result,
-                  uint32_t *__restrict__ slot_out, int32_t *status) {
+                  unsigned long long *counter, unsigned long long epoch, const uint8_t *keys,
+                  const uint32_t *slots, uint64_t n, const int64_t *key_off,
+                  const int32_t *hit, uint32_t R, int32_t *result,
+                  uint32_t *slot_out, int32_t *status) {
     __shared__ unsigned long long block_claims;
     if (threadIdx.x == 0) block_claims = 0;
     __syncthreads();
-    pk::pdl_launch_dependents();
-    pk::pdl_wait();
+    pk::pdl_wait(table, counter, keys, slots, key_off, hit, result, slot_out, status);
     const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t lane = threadIdx.x & 31;
     int64_t a = 0, b = 0, first = 0;
     if (r < R) {  // uniform per warp
-        a = __ldg(key_off + r);
-        b = __ldg(key_off + r + 1);
+        a = __ldcg(key_off + r);
+        b = __ldcg(key_off + r + 1);
         if ((uint64_t)b > n) b = (int64_t)n;
-        const int64_t h0 = __ldg(hit + r);
+        const int64_t h0 = __ldcg(hit + r);
         first = a + (h0 > 0 ? h0 : 0);
     }
     unsigned long long cnt = 0;
@@ -690,8 +690,8 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
     uint4 buf = make_uint4(0, 0, 0, 0);  // key and slot of index cursor + lane
     uint32_t buf_slot = 0;
     if (first + lane < b) {
-        buf = ld_nc_v4(keys + 32 * (first + lane));
-        buf_slot = __ldg(slots + first + lane);
+        buf = ld_cg_v4(keys + 32 * (first + lane));
+        buf_slot = __ldcg(slots + first + lane);
     }
     for (;;) {
         const uint32_t F = __ballot_sync(kFull, !s.pending);
@@ -715,8 +715,8 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
             buf_slot = __shfl_sync(kFull, buf_slot, (lane + nF) & 31);
             cursor += nF;
             if (lane + nF >= 32 && cursor + lane < b) {
-                buf = ld_nc_v4(keys + 32 * (cursor + lane));
-                buf_slot = __ldg(slots + cursor + lane);
+                buf = ld_cg_v4(keys + 32 * (cursor + lane));
+                buf_slot = __ldcg(slots + cursor + lane);
             }
         }
         const uint32_t P = __ballot_sync(kFull, s.pending);
@@ -732,6 +732,7 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
             if (res < 0) set_status(status, res);
         }
     }
+    pk::pdl_launch_dependents();
     count_claims(&block_claims, claims, counter);
 }
 
@@ -750,21 +751,20 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
 // One warp per request, refilled from a register buffer as k_lookup_req.
 __global__ void __launch_bounds__(256, 3)
 k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
-                   unsigned long long *counter, unsigned long long epoch, const uint8_t *__restrict__ keys,
-                   const uint32_t *__restrict__ new_slots, const int64_t *__restrict__ key_off, uint32_t R,
-                   uint64_t key_capacity, uint32_t *__restrict__ slots, int32_t *__restrict__ hit,
-                   int32_t *__restrict__ result, uint32_t *__restrict__ slot_out, int32_t *status) {
+                   unsigned long long *counter, unsigned long long epoch, const uint8_t *keys,
+                   const uint32_t *new_slots, const int64_t *key_off, uint32_t R,
+                   uint64_t key_capacity, uint32_t *slots, int32_t *hit,
+                   int32_t *result, uint32_t *slot_out, int32_t *status) {
     __shared__ unsigned long long block_claims;
     if (threadIdx.x == 0) block_claims = 0;
     __syncthreads();
-    pk::pdl_launch_dependents();
-    pk::pdl_wait();
+    pk::pdl_wait(table, counter, keys, new_slots, key_off, slots, hit, result, slot_out, status);
     const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t lane = threadIdx.x & 31;
     int64_t a = 0, b = 0;
     if (r < R) {  // uniform per warp
-        a = __ldg(key_off + r);
-        b = __ldg(key_off + r + 1);
+        a = __ldcg(key_off + r);
+        b = __ldcg(key_off + r + 1);
         if ((uint64_t)b > key_capacity) b = (int64_t)key_capacity;
     }
     unsigned long long cnt = 0;
@@ -780,8 +780,8 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
     uint4 buf = make_uint4(0, 0, 0, 0);  // key and slot of index cursor + lane
     uint32_t buf_slot = 0;
     if (a + lane < b) {
-        buf = ld_nc_v4(keys + 32 * (a + lane));
-        buf_slot = __ldg(new_slots + a + lane);
+        buf = ld_cg_v4(keys + 32 * (a + lane));
+        buf_slot = __ldcg(new_slots + a + lane);
     }
     for (;;) {
         const uint32_t F = __ballot_sync(kFull, !s.pending);
@@ -806,8 +806,8 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
             buf_slot = __shfl_sync(kFull, buf_slot, (lane + nF) & 31);
             cursor += nF;
             if (lane + nF >= 32 && cursor + lane < b) {
-                buf = ld_nc_v4(keys + 32 * (cursor + lane));
-                buf_slot = __ldg(new_slots + cursor + lane);
+                buf = ld_cg_v4(keys + 32 * (cursor + lane));
+                buf_slot = __ldcg(new_slots + cursor + lane);
             }
         }
         const uint32_t P = __ballot_sync(kFull, s.pending);
@@ -830,6 +830,7 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
             }
         }
     }
+    pk::pdl_launch_dependents();  // main work done: release the finalize kernel
     const uint32_t hm = __reduce_min_sync(kFull, first_miss);
     const int64_t h = hm != 0xffffffffu ? (int64_t)hm : (b > a ? b - a : 0);
     __syncwarp();
@@ -846,17 +847,16 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
 // then finds h_r and relabels.
 __global__ void __launch_bounds__(256)
 k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity, unsigned long long *counter,
-               unsigned long long epoch, const uint8_t *__restrict__ keys, const uint32_t *__restrict__ new_slots,
-               const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capacity, uint32_t *__restrict__ slots,
-               int32_t *__restrict__ result, uint32_t *__restrict__ slot_out, int32_t *status) {
+               unsigned long long epoch, const uint8_t *keys, const uint32_t *new_slots,
+               const int64_t *key_off, uint32_t R, uint64_t key_capacity, uint32_t *slots,
+               int32_t *result, uint32_t *slot_out, int32_t *status) {
     __shared__ unsigned long long block_claims;
     if (threadIdx.x == 0) block_claims = 0;
     __syncthreads();
-    pk::pdl_launch_dependents();
-    pk::pdl_wait();
+    pk::pdl_wait(table, counter, keys, new_slots, key_off, slots, result, slot_out, status);
     const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const uint32_t lane = threadIdx.x & 31;
-    const int64_t total = R == 0 ? 0 : __ldg(key_off + R);
+    const int64_t total = R == 0 ? 0 : __ldcg(key_off + R);
     const int64_t end = total < (int64_t)key_capacity ? total : (int64_t)key_capacity;
     unsigned long long cnt = 0;
     if (lane == 0) cnt = ld_volatile_u64(counter);
@@ -867,8 +867,8 @@ k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capa
     ProbeKey s;
     s.pending = false;
     if (e < end) {
-        const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
-        const uint32_t sl = __ldg(new_slots + e);
+        const uint4 key = __ldcg(reinterpret_cast<const uint4 *>(keys + 32 * e));
+        const uint32_t sl = __ldcg(new_slots + e);
         if (is_zero(key))
             res = PK_ERR_RESERVED_KEY;  // the empty marker: never stored, so a miss
         else
@@ -882,6 +882,7 @@ k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capa
         slot_out[e] = out;
         if (lslot == PK_NO_SLOT && res < 0) set_status(status, res);
     }
+    pk::pdl_launch_dependents();
     count_claims(&block_claims, claims, counter);
 }
 
@@ -889,16 +890,16 @@ k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capa
 // it relabelled PK_STORE_SKIPPED, and PK_ERR_ARG reported for a hit at or
 // after h_r whose slot was PK_NO_SLOT.
 __global__ void __launch_bounds__(256)
-k_lookup_store_tail(const int64_t *__restrict__ key_off, uint32_t R, uint64_t key_capacity,
-                    const uint32_t *__restrict__ slots, int32_t *__restrict__ hit, int32_t *__restrict__ result,
-                    uint32_t *__restrict__ slot_out, int32_t *status) {
+k_lookup_store_tail(const int64_t *key_off, uint32_t R, uint64_t key_capacity,
+                    const uint32_t *slots, int32_t *hit, int32_t *result,
+                    uint32_t *slot_out, int32_t *status) {
     pk::pdl_launch_dependents();
-    pk::pdl_wait();
+    pk::pdl_wait(key_off, slots, hit, result, slot_out, status);
     const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const uint32_t lane = threadIdx.x & 31;
     if (r >= R) return;
-    const int64_t a = __ldg(key_off + r);
-    int64_t b = __ldg(key_off + r + 1);
+    const int64_t a = __ldcg(key_off + r);
+    int64_t b = __ldcg(key_off + r + 1);
     if ((uint64_t)b > key_capacity) b = (int64_t)key_capacity;
     int64_t h = b > a ? b - a : 0;
     bool arg = false;
@@ -924,13 +925,13 @@ k_lookup_store_tail(const int64_t *__restrict__ key_off, uint32_t R, uint64_t ke
 // PRESENT with its slot.  In range mode, entries past key_off[R] (not keys
 // of this batch) are skipped.
 __global__ void __launch_bounds__(256)
-k_store_finalize(const pk_entry *table, uint64_t n, const int64_t *__restrict__ key_off, uint32_t R,
-                 int32_t *__restrict__ result, uint32_t *__restrict__ slot_out) {
+k_store_finalize(const pk_entry *table, uint64_t n, const int64_t *key_off, uint32_t R,
+                 int32_t *result, uint32_t *slot_out) {
     pk::pdl_launch_dependents();
-    pk::pdl_wait();
+    pk::pdl_wait(table, key_off, result, slot_out);
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (e >= n) return;
-    if (key_off && (int64_t)e >= (R > 0 ? __ldg(key_off + R) : 0)) {
+    if (key_off && (int64_t)e >= (R > 0 ? __ldcg(key_off + R) : 0)) {
         result[e] = PK_STORE_SKIPPED;
         slot_out[e] = PK_NO_SLOT;
         return;
@@ -967,17 +968,17 @@ static __device__ __align__(256) NoallocScratch g_noalloc_scratch;
 
 // Count the occupied entries and find the latest call number in the table.
 __global__ void __launch_bounds__(256)
-k_noalloc_scan(const pk_entry *__restrict__ table, uint64_t capacity, NoallocScratch *sc) {
+k_noalloc_scan(const pk_entry *table, uint64_t capacity, NoallocScratch *sc) {
     __shared__ unsigned long long blk_count, blk_epoch;
     if (threadIdx.x == 0) blk_count = blk_epoch = 0;
     __syncthreads();
     unsigned long long cnt = 0, ep = 0;
     for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < capacity;
          i += (uint64_t)gridDim.x * blockDim.x) {
-        const uint4 k = __ldg(reinterpret_cast<const uint4 *>(table[i].k));
+        const uint4 k = __ldcg(reinterpret_cast<const uint4 *>(table[i].k));
         if (!is_zero(k)) {
             ++cnt;
-            const unsigned long long e = __ldg(&table[i].epoch);
+            const unsigned long long e = __ldcg(&table[i].epoch);
             ep = e > ep ? e : ep;
         }
     }
@@ -995,9 +996,9 @@ k_noalloc_scan(const pk_entry *__restrict__ table, uint64_t capacity, NoallocScr
 // positions go to scratch.
 __global__ void __launch_bounds__(256, 4)
 k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity, NoallocScratch *sc,
-                const uint8_t *__restrict__ keys, const uint32_t *__restrict__ slots, uint64_t n,
-                const int64_t *__restrict__ key_off, const int32_t *__restrict__ hit, uint32_t R,
-                int32_t *__restrict__ result, uint32_t *__restrict__ slot_out, int32_t *status) {
+                const uint8_t *keys, const uint32_t *slots, uint64_t n,
+                const int64_t *key_off, const int32_t *hit, uint32_t R,
+                int32_t *result, uint32_t *slot_out, int32_t *status) {
     __shared__ unsigned long long block_claims;
     if (threadIdx.x == 0) block_claims = 0;
     __syncthreads();
@@ -1015,7 +1016,7 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
     ProbeKey s;
     s.pending = false;
     if (active) {
-        const uint4 key = __ldg(reinterpret_cast<const uint4 *>(keys + 32 * e));
+        const uint4 key = __ldcg(reinterpret_cast<const uint4 *>(keys + 32 * e));
         const uint32_t sl = slots[e];
         if (claimable(key, sl, res)) probe_start(s, key, e, mask, sl);
     }
@@ -1035,8 +1036,8 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
 }
 
 __global__ void __launch_bounds__(256)
-k_noalloc_finalize(const pk_entry *table, const NoallocScratch *sc, uint64_t n, int32_t *__restrict__ result,
-                   uint32_t *__restrict__ slot_out) {
+k_noalloc_finalize(const pk_entry *table, const NoallocScratch *sc, uint64_t n, int32_t *result,
+                   uint32_t *slot_out) {
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (e >= n || result[e] != PK_STORE_PENDING) return;
     const unsigned long long w = *reinterpret_cast<const unsigned long long *>(&table[sc->pos[e]].slot);

@@ -188,3 +188,35 @@ def test_empty_batch():
     assert hit.cpu().tolist() == [0, 0, 0]
     assert kt.entries() == 0
     kt.close()
+
+
+@pytest.mark.parametrize("name", ["long_context", "multi_adapter"])
+def test_store_reads_the_lookup_it_follows(name):
+    """pk_lookup then pk_store in range mode as the last two calls, with the
+    h_r buffer pre-filled with zeros: the store must act on the lookup's h_r
+    (its kernels start while the lookup's are still running)."""
+    from paper_2609_38706_gb300 import pk
+    wl = W.reduced(name)
+    kt, d = seeded(wl)
+    b = wl.batch
+    key_off, keys = kt.derive(b.tokens, b.tok_off, b.desc_idx, d)
+    snap = kt.save()
+    N = keys.shape[0]
+    new_slots = torch.arange(N, dtype=torch.int32, device="cuda") + 777
+    ko = key_off.cpu().numpy()
+    r = oracle_step(wl, keys.cpu().numpy()[: int(ko[-1])], ko, new_slots.cpu().numpy()[: int(ko[-1])].astype(np.uint32),
+                    O.DictTable)
+    for _ in range(4):
+        kt.load(snap)
+        hit = torch.zeros(key_off.numel() - 1, dtype=torch.int32, device="cuda")
+        slots = torch.empty(N, dtype=torch.int32, device="cuda")
+        res = torch.full((N,), -55, dtype=torch.int32, device="cuda")
+        so = torch.empty(N, dtype=torch.int32, device="cuda")
+        torch.cuda.synchronize()
+        pk.pk_lookup(kt.ctx, keys, key_off, hit, slots, kt.status, kt.stream)
+        pk.pk_store(kt.ctx, keys, new_slots, res, so, kt.status, key_off, hit, kt.stream)
+        torch.cuda.synchronize()
+        kt.check("lookup, store")
+        assert np.array_equal(hit.cpu().numpy(), r[0])
+        assert np.array_equal(res.cpu().numpy()[: int(ko[-1])], r[2])
+    kt.close()
