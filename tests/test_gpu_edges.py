@@ -219,8 +219,8 @@ def test_descriptor_digest_device_equals_host_and_oracle():
 
 @pytest.mark.parametrize("R,C", [(9000, 16), (5000, 7)])
 def test_many_requests_span_scan_tiles_and_parts(R, C):
-    """More requests than one scan tile (4096) and enough chunks for the
-    overlapped multi-part derivation; ragged lengths and empty requests."""
+    """More requests than one scan tile (4096), many chunks; ragged lengths
+    and empty requests."""
     rng = np.random.default_rng(R + C)
     lens = rng.integers(0, 40 * C, R)
     lens[::13] = 0
