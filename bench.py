@@ -266,10 +266,25 @@ def main():
 
     # ---- resident inputs and outputs ----
     R, N_cap = b.R, b.n_tokens // C
-    tokens_h = torch.from_numpy(b.tokens).pin_memory()
-    tok_off_h = torch.from_numpy(b.tok_off).pin_memory()
-    desc_idx_h = torch.from_numpy(b.desc_idx.view(np.int32)).pin_memory()
-    tokens_d, tok_off_d, desc_idx_d = tokens_h.to(dev), tok_off_h.to(dev), desc_idx_h.to(dev)
+    # The step's inputs in one pinned staging buffer, and a device buffer of the same layout (request
+    # offsets, descriptor indices, tokens), so that a step moves them with one host->device copy; the
+    # results likewise in one device buffer (h_r, slots, store results, output slots) and one copy back.
+    def align(n, a=256):
+        return (n + a - 1) // a * a
+    o_desc = align(8 * (R + 1))
+    o_tok = o_desc + align(4 * R)
+    in_bytes = o_tok + 4 * b.n_tokens
+    in_h = torch.zeros(in_bytes, dtype=torch.uint8).pin_memory()
+    in_h[: 8 * (R + 1)].view(torch.int64).copy_(torch.from_numpy(b.tok_off))
+    in_h[o_desc: o_desc + 4 * R].view(torch.int32).copy_(torch.from_numpy(b.desc_idx.view(np.int32)))
+    in_h[o_tok:].view(torch.int32).copy_(torch.from_numpy(b.tokens))
+    in_d = in_h.to(dev)
+
+    def inputs(buf):
+        return (buf[o_tok:].view(torch.int32), buf[: 8 * (R + 1)].view(torch.int64),
+                buf[o_desc: o_desc + 4 * R].view(torch.int32))
+    tokens_h, tok_off_h, desc_idx_h = inputs(in_h)
+    tokens_d, tok_off_d, desc_idx_d = inputs(in_d)
     descs = pk.Descriptors(wl.descriptors)
     # one pinned staging buffer: D+1 int64 offsets, then the encodings; the key-derivation launch reads
     # it in place, so it is rewritten only after the previous step has completed
@@ -282,15 +297,14 @@ def main():
     digests_d = torch.zeros((descs.count, 32), dtype=torch.uint8, device=dev)
     key_off_d = torch.empty(R + 1, dtype=torch.int64, device=dev)
     keys_d = torch.empty((N_cap, 32), dtype=torch.uint8, device=dev)
-    hit_d = torch.empty(R, dtype=torch.int32, device=dev)
-    slots_d = torch.empty(N_cap, dtype=torch.int32, device=dev)
     new_slots_d = torch.arange(N_cap, dtype=torch.int32, device=dev) + (1 << 30)
-    result_d = torch.empty(N_cap, dtype=torch.int32, device=dev)
-    slot_out_d = torch.empty(N_cap, dtype=torch.int32, device=dev)
-    hit_h = torch.empty(R, dtype=torch.int32).pin_memory()
-    slots_h = torch.empty(N_cap, dtype=torch.int32).pin_memory()
-    result_h = torch.empty(N_cap, dtype=torch.int32).pin_memory()
-    slot_out_h = torch.empty(N_cap, dtype=torch.int32).pin_memory()
+    out_d = torch.empty(R + 3 * N_cap, dtype=torch.int32, device=dev)
+    out_h = torch.empty(R + 3 * N_cap, dtype=torch.int32).pin_memory()
+
+    def outputs(buf):
+        return buf[:R], buf[R: R + N_cap], buf[R + N_cap: R + 2 * N_cap], buf[R + 2 * N_cap:]
+    hit_d, slots_d, result_d, slot_out_d = outputs(out_d)
+    hit_h, slots_h, result_h, slot_out_h = outputs(out_h)
     status = kt.status
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     ctx = kt.ctx
@@ -376,14 +390,9 @@ def main():
             pk.pk_lookup_store(ctx, keys_d, new_slots_d, key_off_d, hit_d, slots_d, result_d, slot_out_d,
                                status)
         else:
-            tokens_d.copy_(tokens_h, non_blocking=True)
-            tok_off_d.copy_(tok_off_h, non_blocking=True)
-            desc_idx_d.copy_(desc_idx_h, non_blocking=True)
+            in_d.copy_(in_h, non_blocking=True)
             core()
-        hit_h.copy_(hit_d, non_blocking=True)
-        slots_h.copy_(slots_d, non_blocking=True)
-        result_h.copy_(result_d, non_blocking=True)
-        slot_out_h.copy_(slot_out_d, non_blocking=True)
+        out_h.copy_(out_d, non_blocking=True)
 
     e2e_ms = {True: [], False: []}
     for in_place in (True, False):
@@ -401,8 +410,8 @@ def main():
         raise RuntimeError("device status after e2e steps")
     if not np.array_equal(hit_h.numpy(), hit_ref):
         raise RuntimeError("e2e hit lengths differ from the device-resident run")
-    h2d = tokens_h.numel() * 4 + tok_off_h.numel() * 8 + desc_idx_h.numel() * 4 + off_bytes + n_enc
-    d2h = (hit_h.numel() + slots_h.numel() + result_h.numel() + slot_out_h.numel()) * 4
+    h2d = in_bytes + off_bytes + n_enc
+    d2h = out_h.numel() * 4
 
     total_ms = float(np.sum(step_ms))
     e2e_total = float(np.sum(e2e_ms[False]))
@@ -459,8 +468,8 @@ def main():
                            "peak_source": peaks["source"]},
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_total / args.steps,
-                "h2d": "pinned host -> device copies of tokens, offsets and descriptor indices (descriptor "
-                       "encodings read in place); results copied back",
+                "h2d": "one pinned host -> device copy of tokens, request offsets and descriptor indices "
+                       "(descriptor encodings read in place); one copy of the results back",
                 "in_place_reads": {"value": tokens_per_step * args.steps * world / (e2e_inplace_total / 1e3),
                                    "ms_per_step": e2e_inplace_total / args.steps,
                                    "note": "all inputs read by the kernels from pinned host memory"}},
