@@ -188,6 +188,23 @@ def workload_config(wl, args) -> dict:
             "between_steps": "L2 flushed (256 MiB write) and table restored to its seeded snapshot, untimed"}
 
 
+def max_over_ranks(times_ms, world: int, device=None):
+    """The job's times: each the maximum over the ranks (replicas) of the
+    local time; identity for one process."""
+    if world <= 1:
+        return [float(x) for x in times_ms]
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x) for x in times_ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t.cpu()]
+
+
+def job_rate(units_per_step: float, steps: int, world: int, total_ms: float) -> float:
+    """Whole-job throughput: the units all ranks processed over the slowest rank's time."""
+    return units_per_step * steps * world / (total_ms / 1e3)
+
+
 def run_reference(args, rank: int, world: int) -> None:
     if rank != 0:
         return
@@ -416,13 +433,10 @@ def main():
     total_ms = float(np.sum(step_ms))
     e2e_total = float(np.sum(e2e_ms[False]))
     e2e_inplace_total = float(np.sum(e2e_ms[True]))
-    if world > 1:
-        t = torch.tensor([total_ms, e2e_total, e2e_inplace_total], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms, e2e_total, e2e_inplace_total = float(t[0]), float(t[1]), float(t[2])
+    total_ms, e2e_total, e2e_inplace_total = max_over_ranks([total_ms, e2e_total, e2e_inplace_total], world, dev)
     tokens_per_step = wl.tokens_keyed()
-    value = tokens_per_step * args.steps * world / (total_ms / 1e3)
-    e2e_value = tokens_per_step * args.steps * world / (e2e_total / 1e3)
+    value = job_rate(tokens_per_step, args.steps, world, total_ms)
+    e2e_value = job_rate(tokens_per_step, args.steps, world, e2e_total)
 
     peaks = load_peaks()
     c_dig, c_chain = compressions(n_keys, C)
@@ -444,8 +458,8 @@ def main():
         "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
         "config": workload_config(wl, args),
-        "lookups_per_s": n_keys * args.steps * world / (total_ms / 1e3),
-        "requests_per_s": R * args.steps * world / (total_ms / 1e3),
+        "lookups_per_s": job_rate(n_keys, args.steps, world, total_ms),
+        "requests_per_s": job_rate(R, args.steps, world, total_ms),
         "phase_ms": {"a0_host": float(np.mean(a0_ms)), "descriptors_and_keys": float(np.mean(derive_ms)),
                      "lookup_and_store": float(np.mean(table_ms)),
                      "note": "separate steps with events between the phases (each event also ends the "
@@ -470,7 +484,7 @@ def main():
                 "ms_per_step": e2e_total / args.steps,
                 "h2d": "one pinned host -> device copy of tokens, request offsets and descriptor indices "
                        "(descriptor encodings read in place); one copy of the results back",
-                "in_place_reads": {"value": tokens_per_step * args.steps * world / (e2e_inplace_total / 1e3),
+                "in_place_reads": {"value": job_rate(tokens_per_step, args.steps, world, e2e_inplace_total),
                                    "ms_per_step": e2e_inplace_total / args.steps,
                                    "note": "all inputs read by the kernels from pinned host memory"}},
         # per step: chunk offsets, chunk+descriptor digests, chain; lookup-and-store (one kernel of
