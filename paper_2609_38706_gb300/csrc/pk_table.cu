@@ -35,10 +35,13 @@ __device__ __forceinline__ uint64_t home_of(const uint4 &k) {
     return ((uint64_t)k.y << 32) | k.x;  // bytes 0..7, little-endian
 }
 
-// Loads that observe concurrent writes of the same kernel.
-__device__ __forceinline__ uint4 ld_volatile_v4(const uint32_t *p) {
+// Reads of table entries that other warps of the same kernel may be claiming:
+// L2 reads (no L1 copy), issued each time they are asked for.  They only
+// guide the probe: every decision that could race is taken by a CAS, and a
+// torn read is re-read atomically (examine).
+__device__ __forceinline__ uint4 ld_l2_v4(const uint32_t *p) {
     uint4 v;
-    asm volatile("ld.volatile.global.v4.u32 {%0, %1, %2, %3}, [%4];"
+    asm volatile("ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%4];"
                  : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                  : "l"(p));
     return v;
@@ -393,7 +396,7 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
             (cur.z == 0 || cur.z == key.z) && (cur.w == 0 || cur.w == key.w))
             cur = atomicCAS(kp, key, key);
         if (same(cur, key)) {
-            const uint4 m = ld_volatile_v4(&ent->slot);  // slot, owner, epoch in one read
+            const uint4 m = ld_l2_v4(&ent->slot);  // slot, owner, epoch in one read
             const unsigned long long ep = ((unsigned long long)m.w << 32) | m.z;
             if (ep != 0ull && ep != epoch) {  // inserted by an earlier call
                 const uint32_t sl = m.x;
@@ -487,7 +490,7 @@ __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, Probe
 #pragma unroll
         for (uint32_t u = 0; u < kWin; ++u) {  // entries before the sequence start are not read
             v[u] = make_uint4(0, 0, 0, 0);
-            if (u < win && (rd.j > 0 || u >= j0)) v[u] = ld_volatile_v4(grp[u].k);
+            if (u < win && (rd.j > 0 || u >= j0)) v[u] = ld_l2_v4(grp[u].k);
         }
 #pragma unroll
         for (uint32_t u = 0; u < kWin; ++u) {
