@@ -268,7 +268,7 @@ struct DescWork {
 __global__ void __launch_bounds__(kDigestBlock)
 k_chunk_digest(const int32_t *tokens, const int64_t *tok_off,
                const int64_t *key_off, uint32_t R, uint32_t C, const __grid_constant__ PadKW pad,
-               uint8_t *keys, const __grid_constant__ DescWork dw, uint32_t r_begin, uint32_t r_end) {
+               uint8_t *keys, const __grid_constant__ DescWork dw) {
     __shared__ uint32_t sK[64], sPad[64];
     __shared__ __align__(16) uint32_t ring[kStages][kDigestBlock][16];
     // The successor (the chain) is released as each block finishes, not at its start: released early,
@@ -289,11 +289,11 @@ k_chunk_digest(const int32_t *tokens, const int64_t *tok_off,
     load_tables(sK, sPad, pad);
     __syncthreads();
     pk::pdl_wait(tokens, tok_off, key_off, keys);
-    if (R == 0 || r_begin >= r_end) return;
-    // the chunks of requests [r_begin, r_end), in tiles of one block, grid-strided
-    const int64_t g_begin = __ldcg(key_off + r_begin), g_end = __ldcg(key_off + r_end);
+    if (R == 0) return;
+    // all chunks, in tiles of one block, grid-strided
+    const int64_t g_end = __ldcg(key_off + R);
     const uint32_t nblocks = gridDim.x - dw.desc_blocks;
-    for (int64_t tile = g_begin + (int64_t)(blockIdx.x - dw.desc_blocks) * kDigestBlock; tile < g_end;
+    for (int64_t tile = (int64_t)(blockIdx.x - dw.desc_blocks) * kDigestBlock; tile < g_end;
          tile += (int64_t)nblocks * kDigestBlock) {
         const int64_t g = tile + threadIdx.x;
         const int64_t g0 = g - (threadIdx.x & 31);
@@ -363,11 +363,11 @@ __device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint32_t (*kw)[
 
 __global__ void __launch_bounds__(2 * kChainLanes)
 k_chain(const int64_t *key_off, const uint32_t *desc_idx,
-        const uint8_t *digests, uint32_t r_begin, uint32_t R, uint32_t D, uint8_t *keys) {
+        const uint8_t *digests, uint32_t R, uint32_t D, uint8_t *keys) {
     __shared__ __align__(16) ChainSmem sm;
     pk::pdl_wait(key_off, desc_idx, digests, keys);  // successor released at the last step (see k_chunk_digest)
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const uint32_t r = r_begin + blockIdx.x * kChainLanes + lane;  // requests [r_begin, R)
+    const uint32_t r = blockIdx.x * kChainLanes + lane;
     int64_t a = 0, n = 0;
     uint32_t di = 0;
     if (r < R) {
@@ -526,15 +526,15 @@ cudaError_t pk_launch_derive_enc(const pk_ctx *ctx, const int32_t *tokens, uint6
     const bool chunks = R > 0 && key_capacity > 0;
     if (!chunks) {
         if (dw.desc_blocks)
-            e = pk_launch(k_chunk_digest, dw.desc_blocks, kDigestBlock, s, tokens, tok_off, (const int64_t *)key_off, R,
-                          C, pad, keys, dw, 0u, 0u);
+            e = pk_launch(k_chunk_digest, dw.desc_blocks, kDigestBlock, s, tokens, tok_off, (const int64_t *)key_off, 0u,
+                          C, pad, keys, dw);
         return e != cudaSuccess ? e : cudaGetLastError();
     }
     e = pk_launch(k_chunk_digest, grid_for(key_capacity, kDigestBlock) + dw.desc_blocks, kDigestBlock, s, tokens,
-                  tok_off, (const int64_t *)key_off, R, C, pad, keys, dw, 0u, R);
+                  tok_off, (const int64_t *)key_off, R, C, pad, keys, dw);
     if (e != cudaSuccess) return e;
     e = pk_launch(k_chain, grid_for(R, kChainLanes), 2 * kChainLanes, s, (const int64_t *)key_off, desc_idx,
-                  (const uint8_t *)digests, 0u, R, D, keys);
+                  (const uint8_t *)digests, R, D, keys);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
