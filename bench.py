@@ -492,6 +492,15 @@ def main():
         "gpu_launches": (3 + (1 if (R >= 1024 or N_cap <= 64 * R) else 2) + 1) * args.steps,
         "clocks": clk,
     }
+    # Two-level variant (request- and worker-level digests): the host cost of one request's digest under a
+    # worker digest computed once, through the C ABI over the batch's R requests.
+    req_descs = pk.Descriptors([wl.descriptors[int(i)] for i in b.desc_idx])
+    worker = pk.pk_worker_digest(wl.descriptors[0])
+    reps = 5
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        pk.pk_request_digests(worker, req_descs)
+    line["two_level_request_digest_us"] = (time.perf_counter() - t0) / (reps * R) * 1e6
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = run_cpu_baseline(wl, args.cpu_seconds)
     if rank == 0:

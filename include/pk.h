@@ -130,6 +130,29 @@ int pk_descriptors_encode(const pk_descriptor *descs, uint32_t D, uint8_t *out, 
 /* Host.  d = SHA-256(enc(canonical descriptor)) (Eq. 3, H over enc). */
 int pk_descriptor_digest(const pk_descriptor *desc, uint8_t out[32]);
 
+/* Host.  Two-level variant: the worker-level and request-level halves of the
+ * descriptor bound through separate digests (Sec. 2.2), the worker half
+ * digested once over resolved values (Sec. 5.3, worker-level digest), the
+ * request half inert when it is empty (Sec. 5.3, request-level tags):
+ *   pk_worker_digest:  d_w = SHA-256(enc_w), enc_w = LE32(4) || (LE32(len) ||
+ *                      bytes) for model id, weight precision, weight version,
+ *                      KV format (canonicalised as above); the descriptor's
+ *                      adapter, salt and appended dimensions are ignored.
+ *   pk_request_digest: d = d_w (worker, 32 bytes) when the descriptor has no
+ *                      adapter, no salt and no appended dimension (such a
+ *                      request keys exactly as the worker-only chain), else
+ *                      d = SHA-256(d_w || SHA-256(enc_q)), enc_q = LE32(2 +
+ *                      n_extra) || (LE32(len) || bytes) for adapter id, salt,
+ *                      appended dimensions; the worker fields are ignored.
+ * d replaces the single-digest d of pk_descriptor_digest as the digest of
+ * pk_derive_keys.  Errors: PK_ERR_ARG, PK_ERR_UNRESOLVED (worker),
+ * PK_ERR_FIELD_TOO_LONG. */
+int pk_worker_digest(const pk_descriptor *desc, uint8_t out[32]);
+int pk_request_digest(const uint8_t worker[32], const pk_descriptor *desc, uint8_t out[32]);
+/* Host.  pk_request_digest for n descriptors of one worker: out[j*32, j*32+32)
+ * for descs[j]; stops at the first error (its code is returned). */
+int pk_request_digests(const uint8_t worker[32], const pk_descriptor *descs, uint32_t n, uint8_t *out);
+
 /* Device.  digests_dev[j] = SHA-256(enc_dev[enc_off_dev[j], enc_off_dev[j+1]))
  * for j < D: the descriptor digests d of a batch (Eq. 3, H over enc), from
  * encodings produced by pk_descriptors_encode and copied to the device.

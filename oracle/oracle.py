@@ -272,6 +272,62 @@ def descriptor_digest(desc: Mapping) -> bytes:
     return sha256(enc(canonicalize(desc)))
 
 
+# ---------------------------------------------------------------------------
+# Two-level variant.  Sec. 2.2: adapter identity and sharing domain (salt) are
+# request-level, weight precision, weight version and KV representation
+# worker-level, and the contract binds the two levels through separate
+# digests.  Sec. 5.3: the worker-level digest is computed once at startup over
+# the resolved values and folded into the model identity; the request-level
+# binding is inert for a request carrying neither adapter nor salt, which then
+# keys exactly as without it, and the two halves compose independently.  Both
+# halves are serialised by the same enc and reduced by the same H.
+# ---------------------------------------------------------------------------
+WORKER_FIELDS = ("model_id", "weight_precision", "weight_version", "kv_format")
+REQUEST_FIELDS = ("adapter_id", "salt")
+
+
+def worker_half(desc: Mapping) -> tuple[bytes, ...]:
+    """The canonical worker-level identities (model id folded in with them;
+    the request fields are not read)."""
+    worker_only = {n: desc.get(n, b"") for n in WORKER_FIELDS}
+    c = dict(zip(REGISTRY_V1, canonicalize(worker_only)))
+    return tuple(c[n] for n in WORKER_FIELDS)
+
+
+def request_half(desc: Mapping) -> tuple[bytes, ...]:
+    """The request-level identities: adapter, salt, then appended dimensions
+    (opaque bytes; the worker fields are not read)."""
+    fields = [_as_bytes(desc.get(n, b"")) for n in REQUEST_FIELDS]
+    fields += [_as_bytes(v) for v in (desc.get("extra", ()) or ())]
+    for v in fields:
+        if len(v) > MAX_FIELD_BYTES:
+            raise OracleError(PK_ERR_FIELD_TOO_LONG, "request field")
+    return tuple(fields)
+
+
+def worker_digest(desc: Mapping) -> bytes:
+    """d_w = H(enc(worker half))."""
+    return sha256(enc(worker_half(desc)))
+
+
+def request_digest(d_w: bytes, desc: Mapping) -> bytes:
+    """The digest a request's keys fold in: d_w itself when the request half
+    is empty (the binding is inert), else H(d_w || H(enc(request half)))."""
+    q = request_half(desc)
+    if all(len(f) == 0 for f in q) and len(q) == len(REQUEST_FIELDS):
+        return bytes(d_w)
+    return sha256(bytes(d_w) + sha256(enc(q)))
+
+
+def two_level_digests(descs: Iterable[Mapping]) -> np.ndarray:
+    """uint8[D][32]: request_digest(worker_digest(d), d) for each descriptor."""
+    descs = list(descs)
+    out = np.zeros((len(descs), 32), np.uint8)
+    for j, d in enumerate(descs):
+        out[j] = np.frombuffer(request_digest(worker_digest(d), d), np.uint8)
+    return out
+
+
 def descriptor_digests(descs: Iterable[Mapping]) -> np.ndarray:
     ds = [descriptor_digest(d) for d in descs]
     if not ds:

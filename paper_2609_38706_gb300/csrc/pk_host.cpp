@@ -82,6 +82,52 @@ int encode(const pk_descriptor *d, std::string *enc) {
     return PK_OK;
 }
 
+// Two-level variant (Sec. 2.2: request-level and worker-level provenance are
+// bound through separate digests; Sec. 5.3: the worker-level digest is taken
+// once over the resolved worker values, and the request-level binding is
+// inert for a request with neither adapter nor salt).  Both halves use enc:
+//   enc_w = LE32(4) || model id, weight precision, weight version, KV format
+//   enc_q = LE32(2 + n_extra) || adapter id, salt, appended dimensions
+int encode_worker(const pk_descriptor *d, std::string *enc) {
+    if (!d) return PK_ERR_ARG;
+    std::string f[4];
+    int rc;
+    if ((rc = opaque(d->model_id, &f[0])) != PK_OK) return rc;
+    if ((rc = canonical_dtype(d->weight_precision, &f[1])) != PK_OK) return rc;
+    if ((rc = opaque(d->weight_version, &f[2])) != PK_OK) return rc;
+    if ((rc = canonical_dtype(d->kv_format, &f[3])) != PK_OK) return rc;
+    enc->clear();
+    put_le32(enc, 4u);
+    for (const auto &s : f) {
+        put_le32(enc, (uint32_t)s.size());
+        enc->append(s);
+    }
+    return PK_OK;
+}
+
+int encode_request(const pk_descriptor *d, std::string *enc, bool *inert) {
+    if (!d) return PK_ERR_ARG;
+    if (d->n_extra && !d->extra) return PK_ERR_ARG;
+    std::string f[2];
+    int rc;
+    if ((rc = opaque(d->adapter_id, &f[0])) != PK_OK) return rc;
+    if ((rc = opaque(d->salt, &f[1])) != PK_OK) return rc;
+    *inert = f[0].empty() && f[1].empty() && d->n_extra == 0;
+    enc->clear();
+    put_le32(enc, 2u + d->n_extra);
+    for (const auto &s : f) {
+        put_le32(enc, (uint32_t)s.size());
+        enc->append(s);
+    }
+    for (uint32_t j = 0; j < d->n_extra; ++j) {
+        std::string x;
+        if ((rc = opaque(d->extra[j], &x)) != PK_OK) return rc;
+        put_le32(enc, (uint32_t)x.size());
+        enc->append(x);
+    }
+    return PK_OK;
+}
+
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? PK_OK : PK_ERR_CUDA; }
 
 }  // namespace
@@ -167,6 +213,41 @@ int pk_descriptor_digest(const pk_descriptor *desc, uint8_t out[32]) {
     const int rc = encode(desc, &enc);
     if (rc != PK_OK) return rc;
     pk::sha256_bytes(reinterpret_cast<const uint8_t *>(enc.data()), enc.size(), out);
+    return PK_OK;
+}
+
+int pk_worker_digest(const pk_descriptor *desc, uint8_t out[32]) {
+    if (!out) return PK_ERR_ARG;
+    std::string enc;
+    const int rc = encode_worker(desc, &enc);
+    if (rc != PK_OK) return rc;
+    pk::sha256_bytes(reinterpret_cast<const uint8_t *>(enc.data()), enc.size(), out);
+    return PK_OK;
+}
+
+int pk_request_digest(const uint8_t worker[32], const pk_descriptor *desc, uint8_t out[32]) {
+    if (!worker || !out) return PK_ERR_ARG;
+    std::string enc;
+    bool inert = false;
+    const int rc = encode_request(desc, &enc, &inert);
+    if (rc != PK_OK) return rc;
+    uint8_t msg[64];
+    std::memcpy(msg, worker, 32);
+    if (inert) {  // keys exactly as the worker-only chain
+        std::memmove(out, msg, 32);
+        return PK_OK;
+    }
+    pk::sha256_bytes(reinterpret_cast<const uint8_t *>(enc.data()), enc.size(), msg + 32);
+    pk::sha256_bytes(msg, 64, out);
+    return PK_OK;
+}
+
+int pk_request_digests(const uint8_t worker[32], const pk_descriptor *descs, uint32_t n, uint8_t *out) {
+    if (n && (!descs || !out)) return PK_ERR_ARG;
+    for (uint32_t j = 0; j < n; ++j) {
+        const int rc = pk_request_digest(worker, descs + j, out + 32ull * j);
+        if (rc != PK_OK) return rc;
+    }
     return PK_OK;
 }
 

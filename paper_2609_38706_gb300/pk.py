@@ -79,6 +79,9 @@ def lib() -> ctypes.CDLL:
             "pk_descriptors_encode": (ctypes.c_int, [ctypes.POINTER(pk_descriptor), _U32, _VP,
                                                      ctypes.c_size_t, _VP]),
             "pk_descriptor_digest": (ctypes.c_int, [ctypes.POINTER(pk_descriptor), _VP]),
+            "pk_worker_digest": (ctypes.c_int, [ctypes.POINTER(pk_descriptor), _VP]),
+            "pk_request_digest": (ctypes.c_int, [_VP, ctypes.POINTER(pk_descriptor), _VP]),
+            "pk_request_digests": (ctypes.c_int, [_VP, ctypes.POINTER(pk_descriptor), _U32, _VP]),
             "pk_digest_descriptors": (ctypes.c_int, [_VP, _VP, _U64, _VP, _U32, _VP, _VP, _VP]),
             "pk_derive_keys": (ctypes.c_int, [_VP, _VP, _U64, _VP, _U32, _VP, _VP, _U32, _VP, _VP, _U64,
                                               _VP, _VP]),
@@ -219,6 +222,39 @@ def pk_descriptor_digest(desc) -> bytes:
     out = (ctypes.c_uint8 * 32)()
     _check(lib().pk_descriptor_digest(d.array, out), "pk_descriptor_digest")
     return bytes(out)
+
+
+def pk_worker_digest(desc) -> bytes:
+    d = _descs([desc]) if isinstance(desc, Mapping) else _descs(desc)
+    out = (ctypes.c_uint8 * 32)()
+    _check(lib().pk_worker_digest(d.array, out), "pk_worker_digest")
+    return bytes(out)
+
+
+def pk_request_digest(worker: bytes, desc) -> bytes:
+    d = _descs([desc]) if isinstance(desc, Mapping) else _descs(desc)
+    w = (ctypes.c_uint8 * 32).from_buffer_copy(bytes(worker))
+    out = (ctypes.c_uint8 * 32)()
+    _check(lib().pk_request_digest(w, d.array, out), "pk_request_digest")
+    return bytes(out)
+
+
+def pk_request_digests(worker: bytes, descs) -> np.ndarray:
+    """uint8[n][32]: pk_request_digest of each descriptor under one worker digest."""
+    d = _descs(descs)
+    w = (ctypes.c_uint8 * 32).from_buffer_copy(bytes(worker))
+    out = np.zeros((max(d.count, 1), 32), np.uint8)
+    _check(lib().pk_request_digests(w, d.array, d.count, _p(out)), "pk_request_digests")
+    return out[: d.count]
+
+
+def two_level_digests(descs) -> np.ndarray:
+    """uint8[D][32]: the two-level digest of each descriptor (its own worker
+    half, then its request half)."""
+    out = np.zeros((len(descs), 32), np.uint8)
+    for j, d in enumerate(descs):
+        out[j] = np.frombuffer(pk_request_digest(pk_worker_digest(d), d), np.uint8)
+    return out
 
 
 def pk_digest_descriptors(ctx: int, enc: torch.Tensor, enc_off: torch.Tensor, digests: torch.Tensor,

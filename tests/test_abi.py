@@ -71,6 +71,48 @@ def test_descriptor_digest_matches_oracle(pk):
         assert pk.pk_descriptor_digest(d) == O.descriptor_digest(d)
 
 
+def test_two_level_digests_match_oracle(pk):
+    rng = np.random.default_rng(15)
+    for _ in range(500):
+        d = _rand_desc(rng)
+        w = pk.pk_worker_digest(d)
+        assert w == O.worker_digest(d)
+        assert pk.pk_request_digest(w, d) == O.request_digest(w, d)
+        other = bytes(rng.integers(0, 256, 32, dtype=np.uint8))  # any worker digest composes
+        assert pk.pk_request_digest(other, d) == O.request_digest(other, d)
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("weight_precision", "auto", -3), ("kv_format", "", -3), ("model_id", "y" * 4097, -4),
+])
+def test_worker_digest_errors_match_oracle(pk, field, value, code):
+    d = {"model_id": "m", "weight_precision": "bf16", "weight_version": "v", "kv_format": "bf16", field: value}
+    with pytest.raises(pk.PKError) as e:
+        pk.pk_worker_digest(d)
+    assert e.value.code == code
+    with pytest.raises(O.OracleError) as e2:
+        O.worker_digest(d)
+    assert e2.value.code == code
+
+
+def test_request_digests_batch(pk):
+    rng = np.random.default_rng(16)
+    descs = [_rand_desc(rng) for _ in range(100)]
+    w = bytes(rng.integers(0, 256, 32, dtype=np.uint8))
+    got = pk.pk_request_digests(w, descs)
+    for j, d in enumerate(descs):
+        assert bytes(got[j]) == O.request_digest(w, d)
+
+
+def test_request_digest_errors(pk):
+    w = bytes(32)
+    with pytest.raises(pk.PKError) as e:
+        pk.pk_request_digest(w, {"salt": "s" * 4097})
+    assert e.value.code == pk.PK_ERR_FIELD_TOO_LONG
+    # the worker fields are not read by the request half: an unresolved dtype is not an error there
+    assert pk.pk_request_digest(w, {"kv_format": "auto", "salt": "s"}) == O.request_digest(w, {"salt": "s"})
+
+
 def test_batch_encode_offsets(pk):
     rng = np.random.default_rng(6)
     descs = [_rand_desc(rng) for _ in range(64)]
