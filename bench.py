@@ -492,6 +492,37 @@ def main():
         "gpu_launches": (3 + (1 if (R >= 1024 or N_cap <= 64 * R) else 2) + 1) * args.steps,
         "clocks": clk,
     }
+    # Store-side omission test (comparison step, pk_compare_pages): 16,384 joined pages of 16 KiB against a
+    # reference set, 1/8 of them absent and 1/4 differing in one byte; HBM-bound.  The 512 MiB of pages are
+    # larger than L2, so no flush between repetitions (a flush's dirty lines would be written back during
+    # the next read).
+    n_pg, pg_bytes = 16384, 16384
+    gen = torch.Generator(device=dev).manual_seed(7)
+    ref_pages = torch.randint(0, 256, (n_pg, pg_bytes), dtype=torch.uint8, device=dev, generator=gen)
+    perm = torch.randperm(n_pg, device=dev, generator=gen)
+    pages = ref_pages[perm].clone()
+    pages[: n_pg // 4, pg_bytes // 2] ^= 1
+    pg_slots = perm.to(torch.int32)
+    pg_slots[n_pg - n_pg // 8:] = -1                        # PK_NO_SLOT
+    verdict = torch.empty(n_pg, dtype=torch.int32, device=dev)
+    counts = torch.zeros(3, dtype=torch.int64, device=dev)
+    cmp_ms = []
+    for it in range(8):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        pk.pk_compare_pages(pg_slots, pages, ref_pages, verdict, counts, status)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if it >= 3:
+            cmp_ms.append(e0.elapsed_time(e1))
+    if kt.take_status() != 0 or counts.tolist() != [8 * (n_pg // 8), 8 * (n_pg - n_pg // 8 - n_pg // 4),
+                                                     8 * (n_pg // 4)]:
+        raise RuntimeError("page comparison counts")
+    present = n_pg - n_pg // 8
+    cmp_bytes = 2 * present * pg_bytes + n_pg * 8
+    cmp_gbs = cmp_bytes / (float(np.mean(cmp_ms)) / 1e3) / 1e9
+    del ref_pages, pages
+
     # Two-level variant (request- and worker-level digests): the host cost of one request's digest under a
     # worker digest computed once, through the C ABI over the batch's R requests.
     req_descs = pk.Descriptors([wl.descriptors[int(i)] for i in b.desc_idx])
@@ -501,6 +532,11 @@ def main():
     for _ in range(reps):
         pk.pk_request_digests(worker, req_descs)
     line["two_level_request_digest_us"] = (time.perf_counter() - t0) / (reps * R) * 1e6
+    line["omission_check_roofline"] = {
+        "bound": "hbm", "kernel": "pk_compare_pages", "achieved": cmp_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+        "frac": cmp_gbs / peaks["hbm_gbs"], "us": float(np.mean(cmp_ms)) * 1e3,
+        "bytes_basis": f"{n_pg} joined pages of {pg_bytes} B ({present} present, each read twice) + 8 B per key",
+        "peak_source": peaks["source"]}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = run_cpu_baseline(wl, args.cpu_seconds)
     if rank == 0:

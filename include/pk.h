@@ -60,6 +60,10 @@ extern "C" {
 #define PK_STORE_INSERTED 1        /* new key; the entry's own slot was stored */
 #define PK_STORE_PRESENT 2         /* key already present (or an earlier duplicate in the batch won) */
 
+#define PK_PAGE_ABSENT 0           /* pk_compare_pages: the key has no reference page */
+#define PK_PAGE_EQUAL 1            /* equal key, equal page bytes */
+#define PK_PAGE_DIFFERS 2          /* equal key, differing page bytes: an omitted binding */
+
 #define PK_NO_SLOT 0xFFFFFFFFu     /* lookup miss; not a storable slot value */
 #define PK_MAX_FIELD_BYTES 4096u
 #define PK_KEY_BYTES 32u           /* one full key k_i */
@@ -247,6 +251,24 @@ int pk_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_dev, ui
 int pk_lookup_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_new_dev, const int64_t *key_off_dev,
                     uint32_t R, uint64_t key_capacity, int32_t *hit_chunks_dev, uint32_t *slots_dev,
                     int32_t *result_dev, uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream);
+
+/* Device.  The comparison step of the store-side differential omission test
+ * (Sec. 6.3, omission detection; Eq. 4): a worker's keys joined to a
+ * reference worker's by pk_lookup on a table holding the reference keys
+ * (slot = index of the reference page), then each joined page compared byte
+ * for byte.
+ *   slots_dev      uint32[n]: the reference page of key j, or PK_NO_SLOT
+ *   pages_dev      n pages of page_bytes (the worker's page of key j)
+ *   ref_pages_dev  n_ref pages of page_bytes
+ *   verdict_dev    OUT int32[n]: PK_PAGE_ABSENT, PK_PAGE_EQUAL or PK_PAGE_DIFFERS
+ *   counts_dev     IN/OUT uint64[3]: counts_dev[v] += keys with verdict v
+ *                  (zero it first for this call's counts)
+ * page_bytes: a positive multiple of 16; page buffers 16-byte aligned.  Every
+ * joined pair is read in full.  Device errors: a slot >= n_ref (PK_ERR_ARG in
+ * *status_dev; that key reads as PK_PAGE_ABSENT). */
+int pk_compare_pages(const uint32_t *slots_dev, const uint8_t *pages_dev, const uint8_t *ref_pages_dev, uint64_t n,
+                     uint64_t n_ref, uint64_t page_bytes, int32_t *verdict_dev, uint64_t *counts_dev,
+                     int32_t *status_dev, pk_stream stream);
 
 /* Checkpoint (the shared store outlives workers, Sec. 2.1).  Asynchronous on
  * `stream`: copies the table and its entry count to dst (device or host

@@ -521,3 +521,34 @@ def seed_table(table, seed_keys: np.ndarray, filler: np.ndarray, target_entries:
             raise OracleError(PK_ERR_ARG, "not enough filler keys")
         table.store(filler[:need], np.arange(n_seed, n_seed + need, dtype=np.uint32))
     return table
+
+
+# ---------------------------------------------------------------------------
+# Store-side differential omission test (Sec. 6.3, omission detection; Eq. 4):
+# a key of one worker that a reference worker also wrote, with differing page
+# bytes, means the binding omits a dimension that changes the cached state.
+# ---------------------------------------------------------------------------
+PAGE_ABSENT, PAGE_EQUAL, PAGE_DIFFERS = 0, 1, 2
+
+
+def compare_pages(slots: np.ndarray, pages: np.ndarray, ref_pages: np.ndarray):
+    """Per key j: PAGE_ABSENT if slots[j] is NO_SLOT, else PAGE_EQUAL or
+    PAGE_DIFFERS for pages[j] against ref_pages[slots[j]].  Returns
+    (verdict int32[n], counts int64[3])."""
+    slots = np.asarray(slots, np.uint32)
+    verdict = np.zeros(slots.size, np.int32)
+    for j, s in enumerate(slots):
+        if int(s) != NO_SLOT:
+            verdict[j] = PAGE_EQUAL if np.array_equal(pages[j], ref_pages[int(s)]) else PAGE_DIFFERS
+    return verdict, np.bincount(verdict, minlength=3).astype(np.int64)
+
+
+def omission_check(ref_keys: np.ndarray, ref_pages: np.ndarray, keys: np.ndarray, pages: np.ndarray):
+    """Join keys to the reference worker's on the 128-bit prefix (the first
+    reference page of a repeated key), then compare_pages."""
+    cap = 2
+    while cap <= ref_keys.shape[0]:
+        cap *= 2
+    t = DictTable(cap)
+    t.store(ref_keys, np.arange(ref_keys.shape[0], dtype=np.uint32))
+    return compare_pages(t.get(keys), pages, ref_pages)

@@ -343,6 +343,19 @@ int pk_lookup_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_
                                           reinterpret_cast<cudaStream_t>(stream)));
 }
 
+int pk_compare_pages(const uint32_t *slots_dev, const uint8_t *pages_dev, const uint8_t *ref_pages_dev, uint64_t n,
+                     uint64_t n_ref, uint64_t page_bytes, int32_t *verdict_dev, uint64_t *counts_dev,
+                     int32_t *status_dev, pk_stream stream) {
+    if (n == 0) return PK_OK;
+    if (!slots_dev || !pages_dev || !verdict_dev || !counts_dev || (n_ref && !ref_pages_dev)) return PK_ERR_ARG;
+    if (page_bytes == 0 || page_bytes % 16 || !aligned16(pages_dev) || !aligned16(ref_pages_dev) ||
+        !aligned(slots_dev, 4) || !aligned(verdict_dev, 4) || !aligned(counts_dev, 8))
+        return PK_ERR_ARG;
+    return cuda_rc(pk_launch_compare_pages(slots_dev, pages_dev, ref_pages_dev, n, n_ref, page_bytes, verdict_dev,
+                                           reinterpret_cast<unsigned long long *>(counts_dev), status_dev,
+                                           reinterpret_cast<cudaStream_t>(stream)));
+}
+
 int pk_table_save(pk_ctx *ctx, void *dst, size_t dst_bytes, pk_stream stream) {
     if (!ctx || !dst) return PK_ERR_ARG;
     const size_t tb = pk_table_bytes(ctx->capacity_log2);

@@ -27,6 +27,7 @@ PK_ERR_PROBE_LIMIT = -6
 PK_ERR_RESERVED_KEY = -7
 PK_ERR_CUDA = -8
 PK_ERR_TOO_LARGE = -9
+PK_PAGE_ABSENT, PK_PAGE_EQUAL, PK_PAGE_DIFFERS = 0, 1, 2
 PK_NOALLOC_MAX_ENTRIES = 1 << 18
 PK_STORE_SKIPPED = 0
 PK_STORE_INSERTED = 1
@@ -93,6 +94,7 @@ def lib() -> ctypes.CDLL:
             "pk_entries": (ctypes.c_int, [_VP, ctypes.POINTER(ctypes.c_uint64), _VP]),
             "pk_store_noalloc": (ctypes.c_int, [ctypes.POINTER(pk_config), _VP, _VP, _U64, _VP, _VP, _U32, _VP, _VP,
                                                 _VP, _VP]),
+            "pk_compare_pages": (ctypes.c_int, [_VP, _VP, _VP, _U64, _U64, _U64, _VP, _VP, _VP, _VP]),
             "pk_table_save": (ctypes.c_int, [_VP, _VP, ctypes.c_size_t, _VP]),
             "pk_table_load": (ctypes.c_int, [_VP, _VP, ctypes.c_size_t, _VP]),
             "pk_strerror": (ctypes.c_char_p, [ctypes.c_int]),
@@ -307,6 +309,14 @@ def pk_lookup_store(ctx: int, keys: torch.Tensor, new_slots: torch.Tensor, key_o
     _check(lib().pk_lookup_store(ctx, _p(keys), _p(new_slots), _p(key_off), R, keys.numel() // 32,
                                  _p(hit_chunks), _p(slots), _p(result), _p(slot_out), _p(status), _s(stream)),
            "pk_lookup_store")
+
+
+def pk_compare_pages(slots: torch.Tensor, pages: torch.Tensor, ref_pages: torch.Tensor, verdict: torch.Tensor,
+                     counts: torch.Tensor, status: torch.Tensor, stream=None) -> None:
+    """pages: uint8 [n, page_bytes]; ref_pages: uint8 [n_ref, page_bytes]; counts: int64[3] (accumulated)."""
+    n, page_bytes = pages.shape
+    _check(lib().pk_compare_pages(_p(slots), _p(pages), _p(ref_pages), n, ref_pages.shape[0], page_bytes,
+                                  _p(verdict), _p(counts), _p(status), _s(stream)), "pk_compare_pages")
 
 
 def pk_table_save(ctx: int, dst: torch.Tensor, stream=None) -> None:

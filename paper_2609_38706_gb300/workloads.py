@@ -25,6 +25,7 @@ from __future__ import annotations
 
 from dataclasses import dataclass, field
 from typing import Optional
+import zlib
 
 import numpy as np
 
@@ -349,3 +350,80 @@ def seed_list(prior_keys: np.ndarray, prior_key_off: np.ndarray, prior_chunks: O
         idx.append(np.arange(a, min(b, a + prior_chunks)))
     idx = np.concatenate(idx) if idx else np.zeros(0, np.int64)
     return prior_keys[idx]
+
+
+# ---------------------------------------------------------------------------
+# Synthetic KV pages for the store-side omission test (sec. 6.3: two workers
+# that differ in one dimension write the same documents into one store).  No
+# model runs here: the bytes of the page of chunk i of a request are a
+# deterministic pseudo-random function of the request's tokens up to the end of
+# chunk i (its prefix, which the state of that chunk depends on) and of the
+# computational dimensions of the worker that wrote it (model id, weight
+# precision, weight version, adapter, KV format).  The salt changes who may
+# reuse state, not the state (sec. 2.2), so it does not enter the bytes.  The
+# seeding uses CRC-32, not the keys' hash.
+# ---------------------------------------------------------------------------
+COMPUTATIONAL_FIELDS = ("model_id", "weight_precision", "weight_version", "adapter_id", "kv_format")
+
+
+def _config_seed(desc: dict) -> int:
+    blob = "\x1f".join(str(desc.get(f, "")) for f in COMPUTATIONAL_FIELDS).encode()
+    return zlib.crc32(blob)
+
+
+def kv_pages(batch: Batch, C: int, desc_of_request, page_bytes: int) -> np.ndarray:
+    """uint8[N_chunks, page_bytes], in key order (request by request, chunk by
+    chunk): the page each full chunk would write.  desc_of_request(r) gives the
+    descriptor of the worker configuration that served request r."""
+    assert page_bytes % 16 == 0
+    pages = []
+    for r in range(batch.R):
+        row = batch.tokens[batch.tok_off[r]:batch.tok_off[r + 1]]
+        cfg = _config_seed(desc_of_request(r))
+        crc = 0
+        for i in range(row.size // C):
+            crc = zlib.crc32(row[i * C:(i + 1) * C].astype("<i4").tobytes(), crc)
+            rng = np.random.default_rng([crc, cfg])
+            pages.append(rng.integers(0, 256, page_bytes, dtype=np.uint8))
+    return np.stack(pages) if pages else np.zeros((0, page_bytes), np.uint8)
+
+
+@dataclass
+class OmissionCase:
+    """Worker A and worker B (A with one dimension changed) serving the same
+    documents; keys are bound with `binding` (the descriptor fields the key
+    covers), pages follow each worker's full configuration."""
+    name: str
+    chunk_tokens: int
+    batch: Batch
+    worker_a: dict
+    worker_b: dict
+    bound_a: dict
+    bound_b: dict
+    pages_a: np.ndarray
+    pages_b: np.ndarray
+
+
+def omission_case(varied: str, omit: Optional[str], seed: int = 5, R: int = 12, T: int = 640, C: int = 64,
+                  page_bytes: int = 256) -> OmissionCase:
+    """`varied`: the dimension in which worker B differs from A; `omit`: the
+    dimension the key binding leaves out (None: the complete binding).  Omitting
+    a field means both workers' key descriptors carry the same fixed value for
+    it."""
+    rng = np.random.default_rng(seed)
+    a = _desc(precision="bf16", version=_hex(rng, 20), adapter="adapter-00", kv="bf16", salt="tenant-a")
+    changed = {"model_id": MODEL_ID + "-v2", "weight_precision": "fp8_e4m3", "weight_version": _hex(rng, 20),
+               "adapter_id": "adapter-01", "kv_format": "fp8_e5m2", "salt": "tenant-b"}
+    b = dict(a, **{varied: changed[varied]})
+    lens = _lengths(rng, R, T, C, True)
+    rows = [rng.integers(0, 32000, int(n), dtype=np.int64).astype(np.int32) for n in lens]
+    toks, off = _pack(rows)
+    batch = Batch(toks, off, np.zeros(R, np.uint32))
+
+    def bound(d):
+        if omit is None:
+            return dict(d)
+        fixed = {"weight_precision": "bf16", "kv_format": "bf16"}.get(omit, "")
+        return dict(d, **{omit: fixed})
+    return OmissionCase(f"vary {varied}, omit {omit}", C, batch, a, b, bound(a), bound(b),
+                        kv_pages(batch, C, lambda r: a, page_bytes), kv_pages(batch, C, lambda r: b, page_bytes))
