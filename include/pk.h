@@ -270,6 +270,32 @@ int pk_compare_pages(const uint32_t *slots_dev, const uint8_t *pages_dev, const 
                      uint64_t n_ref, uint64_t page_bytes, int32_t *verdict_dev, uint64_t *counts_dev,
                      int32_t *status_dev, pk_stream stream);
 
+/* Content identity of large byte buffers (Sec. 5.3: an adapter is bound by an
+ * identity of its contents, every tensor's name, dtype, shape and bytes with
+ * the meaningful configuration fields; Sec. 4.2 leaves the identity function
+ * open as long as it is injective and stable).  One SHA-256 stream over a
+ * tensor is serial, so the bytes are reduced by a fixed-shape tree instead:
+ * every level hashes each 1 KiB block of the level below (the last block
+ * zero-padded; an empty buffer is one zero block), down to one digest, the
+ * "top".  The shape depends only on the byte length, which the tensor
+ * identity binds.
+ *   pk_content_scratch_bytes: device scratch pk_content_digest needs for n_bytes.
+ *   pk_content_digest (device): top_dev (32 bytes) = the tree top of
+ *                     bytes_dev[0, n_bytes); bytes_dev, scratch_dev, top_dev
+ *                     16-byte aligned.  Errors: PK_ERR_ARG (host), PK_ERR_CUDA.
+ *   pk_tensor_identity (host): SHA-256(enc(name, dtype, shape as LE64 each,
+ *                     LE64(n_bytes), top)).
+ *   pk_adapter_identity (host): SHA-256(enc(enc(config fields), tensor
+ *                     identity_0, ..., identity_{n-1})), the tensors in the
+ *                     order given (sort them by name for a stable identity). */
+size_t pk_content_scratch_bytes(uint64_t n_bytes);
+int pk_content_digest(const uint8_t *bytes_dev, uint64_t n_bytes, uint8_t *scratch_dev, size_t scratch_bytes,
+                      uint8_t *top_dev, pk_stream stream);
+int pk_tensor_identity(const pk_bytes *name, const pk_bytes *dtype, const int64_t *shape, uint32_t ndim,
+                       uint64_t n_bytes, const uint8_t top[32], uint8_t out[32]);
+int pk_adapter_identity(const uint8_t *tensor_ids, uint32_t n_tensors, const pk_bytes *config, uint32_t n_config,
+                        uint8_t out[32]);
+
 /* Checkpoint (the shared store outlives workers, Sec. 2.1).  Asynchronous on
  * `stream`: copies the table and its entry count to dst (device or host
  * memory, dst_bytes >= pk_table_bytes(capacity_log2) + 64). */

@@ -552,3 +552,40 @@ def omission_check(ref_keys: np.ndarray, ref_pages: np.ndarray, keys: np.ndarray
     t = DictTable(cap)
     t.store(ref_keys, np.arange(ref_keys.shape[0], dtype=np.uint32))
     return compare_pages(t.get(keys), pages, ref_pages)
+
+
+# ---------------------------------------------------------------------------
+# Content identity (Sec. 5.3: an adapter is bound by an identity of its
+# contents, every tensor's name, dtype, shape and bytes with the meaningful
+# configuration fields; Sec. 4.2: the identity function is open as long as it
+# is injective and stable).  A fixed-shape tree of SHA-256: each level hashes
+# every 1 KiB block of the level below, the last block zero-padded (an empty
+# buffer is one zero block), until one digest remains.
+# ---------------------------------------------------------------------------
+TREE_BLOCK = 1024
+
+
+def tree_level(data: bytes) -> bytes:
+    """The digests of the 1 KiB blocks of data (zero-padded), concatenated."""
+    m = max(1, -(-len(data) // TREE_BLOCK))
+    padded = bytes(data) + bytes(m * TREE_BLOCK - len(data))
+    return b"".join(sha256(padded[i * TREE_BLOCK:(i + 1) * TREE_BLOCK]) for i in range(m))
+
+
+def content_digest(data: bytes) -> bytes:
+    """The tree top of data: levels until one 32-byte digest."""
+    level = tree_level(bytes(data))
+    while len(level) > 32:
+        level = tree_level(level)
+    return level
+
+
+def tensor_identity(name, dtype, shape, n_bytes: int, top: bytes) -> bytes:
+    """H(enc(name, dtype, shape as LE64 each, LE64(n_bytes), top))."""
+    dims = b"".join(int(x).to_bytes(8, "little", signed=True) for x in shape)
+    return sha256(enc([_as_bytes(name), _as_bytes(dtype), dims, int(n_bytes).to_bytes(8, "little"), bytes(top)]))
+
+
+def adapter_identity(tensor_ids, config) -> bytes:
+    """H(enc(enc(config fields), tensor identities in the given order))."""
+    return sha256(enc([enc([_as_bytes(c) for c in config])] + [bytes(t) for t in tensor_ids]))

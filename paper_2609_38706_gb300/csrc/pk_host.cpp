@@ -356,6 +356,67 @@ int pk_compare_pages(const uint32_t *slots_dev, const uint8_t *pages_dev, const 
                                            reinterpret_cast<cudaStream_t>(stream)));
 }
 
+size_t pk_content_scratch_bytes(uint64_t n_bytes) { return (size_t)pk_content_scratch_bytes_impl(n_bytes); }
+
+int pk_content_digest(const uint8_t *bytes_dev, uint64_t n_bytes, uint8_t *scratch_dev, size_t scratch_bytes,
+                      uint8_t *top_dev, pk_stream stream) {
+    if ((n_bytes && !bytes_dev) || !scratch_dev || !top_dev) return PK_ERR_ARG;
+    if (!aligned16(bytes_dev) || !aligned16(scratch_dev) || !aligned16(top_dev)) return PK_ERR_ARG;
+    if (scratch_bytes < pk_content_scratch_bytes_impl(n_bytes)) return PK_ERR_ARG;
+    return cuda_rc(pk_launch_content_digest(bytes_dev, n_bytes, scratch_dev, top_dev,
+                                            reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int pk_tensor_identity(const pk_bytes *name, const pk_bytes *dtype, const int64_t *shape, uint32_t ndim,
+                       uint64_t n_bytes, const uint8_t top[32], uint8_t out[32]) {
+    if (!name || !dtype || (ndim && !shape) || !top || !out) return PK_ERR_ARG;
+    std::string f[2];
+    int rc;
+    if ((rc = opaque(*name, &f[0])) != PK_OK) return rc;
+    if ((rc = opaque(*dtype, &f[1])) != PK_OK) return rc;
+    std::string dims, len;
+    for (uint32_t k = 0; k < ndim; ++k) {
+        put_le32(&dims, (uint32_t)((uint64_t)shape[k] & 0xffffffffu));
+        put_le32(&dims, (uint32_t)((uint64_t)shape[k] >> 32));
+    }
+    put_le32(&len, (uint32_t)(n_bytes & 0xffffffffu));
+    put_le32(&len, (uint32_t)(n_bytes >> 32));
+    std::string enc;
+    put_le32(&enc, 5u);
+    for (const std::string *x : {&f[0], &f[1], &dims, &len}) {
+        put_le32(&enc, (uint32_t)x->size());
+        enc.append(*x);
+    }
+    put_le32(&enc, 32u);
+    enc.append(reinterpret_cast<const char *>(top), 32);
+    pk::sha256_bytes(reinterpret_cast<const uint8_t *>(enc.data()), enc.size(), out);
+    return PK_OK;
+}
+
+int pk_adapter_identity(const uint8_t *tensor_ids, uint32_t n_tensors, const pk_bytes *config, uint32_t n_config,
+                        uint8_t out[32]) {
+    if ((n_tensors && !tensor_ids) || (n_config && !config) || !out) return PK_ERR_ARG;
+    std::string cfg;
+    put_le32(&cfg, n_config);
+    for (uint32_t k = 0; k < n_config; ++k) {
+        std::string x;
+        const int rc = opaque(config[k], &x);
+        if (rc != PK_OK) return rc;
+        put_le32(&cfg, (uint32_t)x.size());
+        cfg.append(x);
+    }
+    std::string enc;
+    put_le32(&enc, 1u + n_tensors);
+    put_le32(&enc, (uint32_t)cfg.size());
+    enc.append(cfg);
+    for (uint32_t t = 0; t < n_tensors; ++t) {
+        put_le32(&enc, 32u);
+        enc.append(reinterpret_cast<const char *>(tensor_ids + 32ull * t), 32);
+    }
+    pk::sha256_bytes(reinterpret_cast<const uint8_t *>(enc.data()), enc.size(), out);
+    return PK_OK;
+}
+
 int pk_table_save(pk_ctx *ctx, void *dst, size_t dst_bytes, pk_stream stream) {
     if (!ctx || !dst) return PK_ERR_ARG;
     const size_t tb = pk_table_bytes(ctx->capacity_log2);

@@ -95,6 +95,11 @@ def lib() -> ctypes.CDLL:
             "pk_store_noalloc": (ctypes.c_int, [ctypes.POINTER(pk_config), _VP, _VP, _U64, _VP, _VP, _U32, _VP, _VP,
                                                 _VP, _VP]),
             "pk_compare_pages": (ctypes.c_int, [_VP, _VP, _VP, _U64, _U64, _U64, _VP, _VP, _VP, _VP]),
+            "pk_content_scratch_bytes": (ctypes.c_size_t, [_U64]),
+            "pk_content_digest": (ctypes.c_int, [_VP, _U64, _VP, ctypes.c_size_t, _VP, _VP]),
+            "pk_tensor_identity": (ctypes.c_int, [ctypes.POINTER(pk_bytes), ctypes.POINTER(pk_bytes), _VP, _U32,
+                                                  _U64, _VP, _VP]),
+            "pk_adapter_identity": (ctypes.c_int, [_VP, _U32, ctypes.POINTER(pk_bytes), _U32, _VP]),
             "pk_table_save": (ctypes.c_int, [_VP, _VP, ctypes.c_size_t, _VP]),
             "pk_table_load": (ctypes.c_int, [_VP, _VP, ctypes.c_size_t, _VP]),
             "pk_strerror": (ctypes.c_char_p, [ctypes.c_int]),
@@ -317,6 +322,42 @@ def pk_compare_pages(slots: torch.Tensor, pages: torch.Tensor, ref_pages: torch.
     n, page_bytes = pages.shape
     _check(lib().pk_compare_pages(_p(slots), _p(pages), _p(ref_pages), n, ref_pages.shape[0], page_bytes,
                                   _p(verdict), _p(counts), _p(status), _s(stream)), "pk_compare_pages")
+
+
+def pk_content_scratch_bytes(n_bytes: int) -> int:
+    return int(lib().pk_content_scratch_bytes(n_bytes))
+
+
+def pk_content_digest(data: torch.Tensor, scratch: torch.Tensor, top: torch.Tensor, stream=None) -> None:
+    """top (uint8[32], device) = tree top of the bytes of `data` (a contiguous device tensor)."""
+    n = data.numel() * data.element_size()
+    _check(lib().pk_content_digest(_p(data), n, _p(scratch), scratch.numel(), _p(top), _s(stream)),
+           "pk_content_digest")
+
+
+def _pkb(b: bytes):
+    buf = ctypes.create_string_buffer(bytes(b), max(len(b), 1))
+    return pk_bytes(ctypes.cast(buf, ctypes.c_void_p), len(b)), buf
+
+
+def pk_tensor_identity(name, dtype, shape, n_bytes: int, top: bytes) -> bytes:
+    nb, k1 = _pkb(name.encode() if isinstance(name, str) else name)
+    db, k2 = _pkb(dtype.encode() if isinstance(dtype, str) else dtype)
+    dims = (ctypes.c_int64 * max(len(shape), 1))(*[int(x) for x in shape])
+    t = (ctypes.c_uint8 * 32).from_buffer_copy(bytes(top))
+    out = (ctypes.c_uint8 * 32)()
+    _check(lib().pk_tensor_identity(ctypes.byref(nb), ctypes.byref(db), dims, len(shape), n_bytes, t, out),
+           "pk_tensor_identity")
+    return bytes(out)
+
+
+def pk_adapter_identity(tensor_ids, config) -> bytes:
+    ids = np.frombuffer(b"".join(bytes(x) for x in tensor_ids), np.uint8) if tensor_ids else np.zeros(32, np.uint8)
+    keep = [_pkb(c.encode() if isinstance(c, str) else c) for c in config]
+    arr = (pk_bytes * max(len(keep), 1))(*[k[0] for k in keep])
+    out = (ctypes.c_uint8 * 32)()
+    _check(lib().pk_adapter_identity(ids.ctypes.data, len(tensor_ids), arr, len(keep), out), "pk_adapter_identity")
+    return bytes(out)
 
 
 def pk_table_save(ctx: int, dst: torch.Tensor, stream=None) -> None:

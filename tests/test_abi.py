@@ -113,6 +113,27 @@ def test_request_digest_errors(pk):
     assert pk.pk_request_digest(w, {"kv_format": "auto", "salt": "s"}) == O.request_digest(w, {"salt": "s"})
 
 
+def test_content_identities_match_oracle(pk):
+    rng = np.random.default_rng(21)
+    for _ in range(200):
+        top = bytes(rng.integers(0, 256, 32, dtype=np.uint8))
+        shape = [int(x) for x in rng.integers(0, 5000, int(rng.integers(0, 5)))]
+        name = bytes(rng.integers(0, 256, int(rng.integers(0, 40)), dtype=np.uint8))
+        n = int(rng.integers(0, 1 << 40))
+        t = pk.pk_tensor_identity(name, "bf16", shape, n, top)
+        assert t == O.tensor_identity(name, "bf16", shape, n, top)
+    ids = [bytes(rng.integers(0, 256, 32, dtype=np.uint8)) for _ in range(7)]
+    cfg = ["r=8", "", "target_modules=q_proj,v_proj"]
+    assert pk.pk_adapter_identity(ids, cfg) == O.adapter_identity(ids, cfg)
+    assert pk.pk_adapter_identity([], []) == O.adapter_identity([], [])
+
+
+def test_content_scratch_bytes(pk):
+    assert pk.pk_content_scratch_bytes(0) == 32 and pk.pk_content_scratch_bytes(1024) == 32
+    assert pk.pk_content_scratch_bytes(1025) == 2 * 32 + 32
+    assert pk.pk_content_scratch_bytes(33 * 1024 + 1) == 34 * 32 + 2 * 32 + 32
+
+
 def test_batch_encode_offsets(pk):
     rng = np.random.default_rng(6)
     descs = [_rand_desc(rng) for _ in range(64)]
