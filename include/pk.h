@@ -272,7 +272,7 @@ int pk_compare_pages(const uint32_t *slots_dev, const uint8_t *pages_dev, const 
 
 /* Content identity of large byte buffers (Sec. 5.3: an adapter is bound by an
  * identity of its contents, every tensor's name, dtype, shape and bytes with
- * the meaningful configuration fields; Sec. 4.2 leaves the identity function
+ * the meaningful configuration fields; Sec. 5.1 leaves the identity function
  * open as long as it is injective and stable).  One SHA-256 stream over a
  * tensor is serial, so the bytes are reduced by a fixed-shape tree instead:
  * every level hashes each 1 KiB block of the level below (the last block

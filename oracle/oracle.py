@@ -557,7 +557,7 @@ def omission_check(ref_keys: np.ndarray, ref_pages: np.ndarray, keys: np.ndarray
 # ---------------------------------------------------------------------------
 # Content identity (Sec. 5.3: an adapter is bound by an identity of its
 # contents, every tensor's name, dtype, shape and bytes with the meaningful
-# configuration fields; Sec. 4.2: the identity function is open as long as it
+# configuration fields; Sec. 5.1: the identity function is open as long as it
 # is injective and stable).  A fixed-shape tree of SHA-256: each level hashes
 # every 1 KiB block of the level below, the last block zero-padded (an empty
 # buffer is one zero block), until one digest remains.

@@ -2,7 +2,7 @@
 // checkpoints) on the GPU.  The paper binds an adapter by an identity of its
 // contents (Sec. 5.3, request-level tags: every tensor's name, dtype, shape
 // and bytes with the meaningful configuration fields) and leaves the identity
-// function open as long as it is injective and stable (Sec. 4.2).  A single
+// function open as long as it is injective and stable (Sec. 5.1).  A single
 // SHA-256 stream over a tensor is serial; this file computes a fixed-shape
 // tree of SHA-256 instead: every level hashes each 1 KiB block of the level
 // below (the last block zero-padded), until one 32-byte digest remains.  The

@@ -1,4 +1,4 @@
-"""Pins of the oracle's content identity (Sec. 5.3 adapter identity; Sec. 4.2:
+"""Pins of the oracle's content identity (Sec. 5.3 adapter identity; Sec. 5.1:
 injective and stable): the fixed-shape SHA-256 tree checked against hashlib
 built by hand for one, two and three levels, its shape, and the properties the
 identity needs (the byte length and every tensor attribute bound)."""
