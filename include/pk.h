@@ -54,6 +54,7 @@ extern "C" {
 #define PK_ERR_RESERVED_KEY (-7)   /* key prefix is all zero (the empty marker), p = 2^-128 */
 #define PK_ERR_CUDA (-8)           /* a CUDA runtime call or launch failed */
 #define PK_ERR_TOO_LARGE (-9)      /* n above PK_NOALLOC_MAX_ENTRIES (pk_store_noalloc only) */
+#define PK_ERR_TIMEOUT (-10)       /* a bounded device-wide wait gave up (pk_evict); table unspecified */
 
 /* Per-entry store results (int32). Negative values are the error codes above. */
 #define PK_STORE_SKIPPED 0         /* not in a miss range (range mode) */
@@ -296,6 +297,80 @@ int pk_tensor_identity(const pk_bytes *name, const pk_bytes *dtype, const int64_
 int pk_adapter_identity(const uint8_t *tensor_ids, uint32_t n_tensors, const pk_bytes *config, uint32_t n_config,
                         uint8_t out[32]);
 
+/* Connector key strings (Sec. 5.3, connector integration).  A connector that
+ * packs its key into a fixed-width text field carries the 128-bit digest as
+ * PK_KEY_STRING_CHARS (22) base64 characters (RFC 4648, Sec. 4: alphabet
+ * A-Z a-z 0-9 + /, big-endian 6-bit groups, the two "=" of padding dropped;
+ * the last character encodes two bits followed by four zero bits) and the
+ * model identity with the worker provenance as a fixed-length hash of the
+ * same form, so the key's length does not depend on the model path.
+ *   pk_key_string (host): out = base64 of key16[0, 16); no terminating NUL.
+ *   pk_model_tag (host): out = pk_key_string of the first 16 bytes of the
+ *                  worker digest d_w of pk_worker_digest (model id, weight
+ *                  precision, weight version, KV format).  Errors as
+ *                  pk_worker_digest.
+ *   pk_key_strings (device): for i < n, row i of out_dev (bytes
+ *                  [i*width, (i+1)*width)) = prefix[0, prefix_len) ||
+ *                  base64 of keys_dev[i*32, i*32+16) || zero bytes up to the
+ *                  row width.  keys_dev: n 32-byte keys of a pk_derive_keys
+ *                  result (16-byte aligned); prefix: host bytes, the same for
+ *                  every row (e.g. the connector's fixed fields and the model
+ *                  tag), may be NULL when prefix_len == 0; out_dev: n*width
+ *                  bytes, 16-byte aligned.  Requires prefix_len + 22 <= width
+ *                  <= PK_KEY_STRING_MAX_WIDTH.  Errors (host, nothing
+ *                  enqueued): PK_ERR_ARG; PK_ERR_CUDA. */
+#define PK_KEY_STRING_CHARS 22u
+#define PK_KEY_STRING_MAX_WIDTH 256u
+int pk_key_string(const uint8_t key16[16], char out[22]);
+int pk_model_tag(const pk_descriptor *desc, char out[22]);
+int pk_key_strings(const uint8_t *keys_dev, uint64_t n, const char *prefix, uint32_t prefix_len, uint32_t width,
+                   char *out_dev, pk_stream stream);
+
+/* Eviction under a fixed budget (Sec. 6.5: provenance separation keeps one
+ * copy per provenance, so a store of fixed size evicts more and thrashes once
+ * the distinct working set exceeds it).  Budget mode keeps one last-use
+ * stamp per table entry in a caller-owned array:
+ *   stamp = (n << 32) | e, n the number of the store call on this context
+ *           (pk_store and pk_lookup_store calls, counted from 1 after
+ *           pk_init; after a pk_table_load the next call number is at least
+ *           2), e the key's index in that call;
+ * each pk_store and pk_lookup_store call raises it to its own for every key
+ * of the call that was in the table at the start of the call, or is stored
+ * by it with a valid slot (in pk_store, every entry with result
+ * PK_STORE_INSERTED or PK_STORE_PRESENT).  pk_lookup reads only and stamps
+ * nothing.  Entries stored before the stamps were attached (or before a
+ * pk_table_load) have stamp 0.
+ *   pk_stamps_bytes:  bytes of the stamp array (8 per entry; 0 if out of range).
+ *   pk_attach_stamps: enable budget mode with stamps_dev (8-byte aligned,
+ *                     >= pk_stamps_bytes) and zero it on `stream`; NULL
+ *                     detaches.
+ *   pk_evict_scratch_bytes: device scratch pk_evict needs (about 8.2 bytes
+ *                     per entry plus 8.5 KiB).
+ *   pk_evict (device): when the table holds more than `budget` entries,
+ *                     remove every entry whose stamp is at most v, the
+ *                     (keep+1)-th largest stamp: the least recently used
+ *                     entries down to `keep` (fewer remain only when stamps
+ *                     tie at v, i.e. unstamped entries).  Otherwise nothing
+ *                     changes.  The slots of the removed entries go to
+ *                     evicted_slots_dev[0, *n_evicted_dev) in unspecified
+ *                     order (evicted_slots_dev: uint32[evicted_cap] or NULL;
+ *                     n_evicted_dev: uint64, 0 when nothing is removed, or
+ *                     NULL); the entry count drops by their number.  Kept
+ *                     entries keep their key, slot and stamp (their positions
+ *                     may change).  Requires stamps attached, keep <= budget,
+ *                     scratch_dev 16-byte aligned with scratch_bytes >=
+ *                     pk_evict_scratch_bytes.  Device errors: more removals
+ *                     than evicted_cap (PK_ERR_ARG; the extra slots are not
+ *                     written); PK_ERR_TIMEOUT (table unspecified).  One
+ *                     cooperative launch; within the budget it returns at
+ *                     once. */
+size_t pk_stamps_bytes(uint32_t capacity_log2);
+int pk_attach_stamps(pk_ctx *ctx, uint64_t *stamps_dev, size_t stamps_bytes, pk_stream stream);
+size_t pk_evict_scratch_bytes(uint32_t capacity_log2);
+int pk_evict(pk_ctx *ctx, uint64_t budget, uint64_t keep, void *scratch_dev, size_t scratch_bytes,
+             uint32_t *evicted_slots_dev, uint64_t evicted_cap, uint64_t *n_evicted_dev, int32_t *status_dev,
+             pk_stream stream);
+
 /* Checkpoint (the shared store outlives workers, Sec. 2.1).  Asynchronous on
  * `stream`: copies the table and its entry count to dst (device or host
  * memory, dst_bytes >= pk_table_bytes(capacity_log2) + 64). */
@@ -304,7 +379,8 @@ int pk_table_save(pk_ctx *ctx, void *dst, size_t dst_bytes, pk_stream stream);
 /* Resume: replace this context's table with one saved by pk_table_save from a
  * context of the same capacity (src: device or host memory, src_bytes >=
  * pk_table_bytes + 64).  Keys and slots are restored exactly; the entries
- * count as inserted before any later store call.  Asynchronous on `stream`. */
+ * count as inserted before any later store call; attached stamps are
+ * zeroed.  Asynchronous on `stream`. */
 int pk_table_load(pk_ctx *ctx, const void *src, size_t src_bytes, pk_stream stream);
 
 /* Device.  The insert-if-absent of pk_store for callers that cannot allocate

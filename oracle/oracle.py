@@ -589,3 +589,132 @@ def tensor_identity(name, dtype, shape, n_bytes: int, top: bytes) -> bytes:
 def adapter_identity(tensor_ids, config) -> bytes:
     """H(enc(enc(config fields), tensor identities in the given order))."""
     return sha256(enc([enc([_as_bytes(c) for c in config])] + [bytes(t) for t in tensor_ids]))
+
+
+# ---------------------------------------------------------------------------
+# Connector key strings (Sec. 5.3, connector integration): a fixed-width text
+# key carries the 128-bit digest as twenty-two base64 characters and the model
+# identity with the worker provenance as a fixed-length hash.  Readings: the
+# alphabet is the standard one of RFC 4648, Sec. 4, without the "=" padding;
+# the fixed-length hash is the first 16 bytes of the worker digest d_w, in
+# the same 22-character form; a key string row is prefix || 22 characters ||
+# zero bytes up to the row width.
+# ---------------------------------------------------------------------------
+B64_ALPHABET = "ABCDEFGHIJKLMNOPQRSTUVWXYZabcdefghijklmnopqrstuvwxyz0123456789+/"
+KEY_STRING_CHARS = 22
+
+
+def base64_encode(data: bytes) -> str:
+    """RFC 4648, Sec. 4: each 24-bit group of input bits (most significant
+    first) is four 6-bit indices into the alphabet; a final group of 8 or 16
+    bits is zero-extended to 12 or 18 bits and followed by "==" or "="."""
+    data = bytes(data)
+    out = []
+    for i in range(0, len(data), 3):
+        group = data[i:i + 3]
+        bits = int.from_bytes(group, "big") << (8 * (3 - len(group)))
+        chars = [B64_ALPHABET[(bits >> (18 - 6 * j)) & 63] for j in range(4)]
+        n_chars = len(group) + 1  # 1 byte -> 2 characters, 2 -> 3, 3 -> 4
+        out.append("".join(chars[:n_chars]) + "=" * (4 - n_chars))
+    return "".join(out)
+
+
+def key_string(prefix16: bytes) -> str:
+    """The 22-character form of a 128-bit key prefix: base64 without "=="."""
+    prefix16 = bytes(prefix16)
+    if len(prefix16) != 16:
+        raise OracleError(PK_ERR_ARG, "a key prefix is 16 bytes")
+    s = base64_encode(prefix16)
+    assert s.endswith("==")
+    return s[:KEY_STRING_CHARS]
+
+
+def model_tag(desc: Mapping) -> str:
+    """The fixed-length hash over the model identity and worker provenance."""
+    return key_string(worker_digest(desc)[:16])
+
+
+def key_strings(keys: np.ndarray, prefix: bytes, width: int) -> np.ndarray:
+    """uint8[n, width]: row i = prefix || key_string(keys[i, :16]) || zeros."""
+    prefix = bytes(prefix)
+    if len(prefix) + KEY_STRING_CHARS > width:
+        raise OracleError(PK_ERR_ARG, "row narrower than prefix + 22 characters")
+    keys = np.asarray(keys, np.uint8).reshape(-1, 32)
+    out = np.zeros((keys.shape[0], width), np.uint8)
+    for i in range(keys.shape[0]):
+        row = prefix + key_string(keys[i, :16].tobytes()).encode("ascii")
+        out[i, :len(row)] = np.frombuffer(row, np.uint8)
+    return out
+
+
+# ---------------------------------------------------------------------------
+# Eviction under a fixed budget (Sec. 6.5: binding provenance keeps one copy
+# per provenance, so a store of fixed size evicts more and thrashes once the
+# distinct working set exceeds it).  Readings: the budget counts entries
+# (chunks); recency is least-recently-used with a last-use stamp
+# (n << 32) | e per entry, n the store call's number on the table and e the
+# key's index in the call; a call uses every key that was in the table at its
+# start or that it stores with a valid slot; eviction runs between calls and,
+# when the table holds more than `budget` entries, removes every entry whose
+# stamp is at most the (keep+1)-th largest (the least recently used, down to
+# `keep`; a group of equal stamps, possible only for never-used entries at
+# stamp 0, goes as a whole).
+# ---------------------------------------------------------------------------
+class BudgetTable:
+    """DictTable plus last-use stamps and the store-call counter."""
+
+    def __init__(self, capacity: int):
+        self.table = DictTable(capacity)
+        self.stamps: dict[bytes, int] = {}
+        self.calls = 0
+
+    def __len__(self):
+        return len(self.table)
+
+    def _use(self, k: bytes, e: int) -> None:
+        s = (self.calls << 32) | e
+        if s > self.stamps.get(k, 0):
+            self.stamps[k] = s
+
+    def store(self, keys: np.ndarray, slots: np.ndarray):
+        """List-mode store; every entry that ends INSERTED or PRESENT is a use."""
+        self.calls += 1
+        res, so = self.table.store(keys, slots)
+        p = prefix128(keys)
+        for e in range(p.shape[0]):
+            if res[e] in (STORE_INSERTED, STORE_PRESENT):
+                self._use(p[e].tobytes(), e)
+        return res, so
+
+    def lookup_store(self, keys: np.ndarray, key_off: np.ndarray, new_slots: np.ndarray):
+        """Lookup, then the store of every miss range (one call)."""
+        self.calls += 1
+        p = prefix128(keys)
+        new_slots = np.asarray(new_slots, np.uint32)
+        present0 = self.table.get(keys) != NO_SLOT if p.shape[0] else np.zeros(0, bool)
+        hit, slots = lookup(self.table, keys, key_off)
+        res, so = store_misses(self.table, keys, key_off, hit, new_slots)
+        for e in range(p.shape[0]):
+            k = p[e].tobytes()
+            if present0[e] or (int(new_slots[e]) != NO_SLOT and k in self.table.map):
+                self._use(k, e)
+        return hit, slots, res, so
+
+    def evict(self, budget: int, keep: int) -> np.ndarray:
+        """Sorted uint32 slots of the removed entries (empty within the budget)."""
+        if keep > budget:
+            raise OracleError(PK_ERR_ARG, "keep > budget")
+        m = self.table.map
+        if len(m) <= budget or len(m) <= keep:
+            return np.zeros(0, np.uint32)
+        v = sorted((self.stamps.get(k, 0) for k in m), reverse=True)[keep]
+        gone = [k for k in m if self.stamps.get(k, 0) <= v]
+        out = np.array(sorted(m[k] for k in gone), np.uint32)
+        for k in gone:
+            del m[k]
+            self.stamps.pop(k, None)
+        return out
+
+    def triples(self):
+        """Sorted (16-byte key, slot, stamp) of every entry."""
+        return sorted((k, s, self.stamps.get(k, 0)) for k, s in self.table.map.items())

@@ -128,6 +128,21 @@ int encode_request(const pk_descriptor *d, std::string *enc, bool *inert) {
     return PK_OK;
 }
 
+// RFC 4648, Sec. 4, without padding: 16 bytes -> 22 characters.
+void base64_16(const uint8_t *in, char *out) {
+    static const char kAlphabet[] = "ABCDEFGHIJKLMNOPQRSTUVWXYZabcdefghijklmnopqrstuvwxyz0123456789+/";
+    uint32_t acc = 0, bits = 0, o = 0;
+    for (int i = 0; i < 16; ++i) {
+        acc = (acc << 8) | in[i];
+        bits += 8;
+        while (bits >= 6) {
+            bits -= 6;
+            out[o++] = kAlphabet[(acc >> bits) & 63u];
+        }
+    }
+    out[o] = kAlphabet[(acc << (6 - bits)) & 63u];  // 2 bits left, 4 zero bits appended
+}
+
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? PK_OK : PK_ERR_CUDA; }
 
 }  // namespace
@@ -153,6 +168,7 @@ int pk_init(pk_ctx **out, const pk_config *cfg, pk_stream stream) {
     c->max_probe = (cfg->max_probe == 0 || cfg->max_probe > c->capacity) ? (uint32_t)c->capacity : cfg->max_probe;
     c->table = static_cast<pk_entry *>(cfg->table_dev);
     c->epoch = 0;
+    c->stamps = nullptr;
     {   // final block of a 4C-byte message when 4C is a multiple of 64: 0x80, zeros, 64-bit bit length
         const uint64_t bits = (uint64_t)cfg->chunk_tokens * 32u;
         const uint32_t m[16] = {0x80000000u, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, (uint32_t)(bits >> 32),
@@ -343,6 +359,67 @@ int pk_lookup_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_
                                           reinterpret_cast<cudaStream_t>(stream)));
 }
 
+size_t pk_stamps_bytes(uint32_t capacity_log2) {
+    if (capacity_log2 < 1 || capacity_log2 > 31) return 0;
+    return (size_t)8 << capacity_log2;
+}
+
+int pk_attach_stamps(pk_ctx *ctx, uint64_t *stamps_dev, size_t stamps_bytes, pk_stream stream) {
+    if (!ctx) return PK_ERR_ARG;
+    if (!stamps_dev) {
+        ctx->stamps = nullptr;
+        return PK_OK;
+    }
+    if (!aligned(stamps_dev, 8) || stamps_bytes < pk_stamps_bytes(ctx->capacity_log2)) return PK_ERR_ARG;
+    if (cudaMemsetAsync(stamps_dev, 0, pk_stamps_bytes(ctx->capacity_log2), reinterpret_cast<cudaStream_t>(stream)) !=
+        cudaSuccess)
+        return PK_ERR_CUDA;
+    ctx->stamps = reinterpret_cast<unsigned long long *>(stamps_dev);
+    return PK_OK;
+}
+
+size_t pk_evict_scratch_bytes(uint32_t capacity_log2) {
+    if (capacity_log2 < 1 || capacity_log2 > 31) return 0;
+    return (size_t)pk_evict_scratch_bytes_impl(1ull << capacity_log2);
+}
+
+int pk_evict(pk_ctx *ctx, uint64_t budget, uint64_t keep, void *scratch_dev, size_t scratch_bytes,
+             uint32_t *evicted_slots_dev, uint64_t evicted_cap, uint64_t *n_evicted_dev, int32_t *status_dev,
+             pk_stream stream) {
+    if (!ctx || !ctx->stamps || keep > budget || !scratch_dev || !aligned16(scratch_dev)) return PK_ERR_ARG;
+    if (scratch_bytes < pk_evict_scratch_bytes_impl(ctx->capacity)) return PK_ERR_ARG;
+    if (!aligned(evicted_slots_dev, 4) || !aligned(n_evicted_dev, 8) || !aligned(status_dev, 4)) return PK_ERR_ARG;
+    return cuda_rc(pk_launch_evict(ctx, budget, keep, scratch_dev, evicted_slots_dev,
+                                   evicted_slots_dev ? evicted_cap : 0,
+                                   reinterpret_cast<unsigned long long *>(n_evicted_dev), status_dev,
+                                   reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int pk_key_string(const uint8_t key16[16], char out[22]) {
+    if (!key16 || !out) return PK_ERR_ARG;
+    base64_16(key16, out);
+    return PK_OK;
+}
+
+int pk_model_tag(const pk_descriptor *desc, char out[22]) {
+    if (!out) return PK_ERR_ARG;
+    uint8_t dw[32];
+    const int rc = pk_worker_digest(desc, dw);
+    if (rc != PK_OK) return rc;
+    base64_16(dw, out);
+    return PK_OK;
+}
+
+int pk_key_strings(const uint8_t *keys_dev, uint64_t n, const char *prefix, uint32_t prefix_len, uint32_t width,
+                   char *out_dev, pk_stream stream) {
+    if (width > PK_KEY_STRING_MAX_WIDTH || prefix_len + PK_KEY_STRING_CHARS > width) return PK_ERR_ARG;
+    if (prefix_len && !prefix) return PK_ERR_ARG;
+    if (n == 0) return PK_OK;
+    if (!keys_dev || !out_dev || !aligned16(keys_dev) || !aligned16(out_dev)) return PK_ERR_ARG;
+    return cuda_rc(pk_launch_key_strings(keys_dev, n, reinterpret_cast<const uint8_t *>(prefix), prefix_len, width,
+                                         reinterpret_cast<uint8_t *>(out_dev), reinterpret_cast<cudaStream_t>(stream)));
+}
+
 int pk_compare_pages(const uint32_t *slots_dev, const uint8_t *pages_dev, const uint8_t *ref_pages_dev, uint64_t n,
                      uint64_t n_ref, uint64_t page_bytes, int32_t *verdict_dev, uint64_t *counts_dev,
                      int32_t *status_dev, pk_stream stream) {
@@ -439,6 +516,7 @@ int pk_table_load(pk_ctx *ctx, const void *src, size_t src_bytes, pk_stream stre
                         cudaMemcpyDefault, s) != cudaSuccess)
         return PK_ERR_CUDA;
     if (ctx->epoch < 1) ctx->epoch = 1;
+    if (ctx->stamps && cudaMemsetAsync(ctx->stamps, 0, 8ull * ctx->capacity, s) != cudaSuccess) return PK_ERR_CUDA;
     return cuda_rc(pk_launch_mark_loaded(ctx, s));
 }
 
@@ -485,6 +563,7 @@ const char *pk_strerror(int code) {
         case PK_ERR_PROBE_LIMIT: return "probe limit reached";
         case PK_ERR_RESERVED_KEY: return "key prefix is the reserved all-zero value";
         case PK_ERR_CUDA: return "CUDA runtime error";
+        case PK_ERR_TIMEOUT: return "a bounded device-wide wait gave up (the table is unspecified)";
         case PK_ERR_TOO_LARGE: return "more entries than the allocation-free store's scratch holds (PK_NOALLOC_MAX_ENTRIES)";
         default: return "unknown status";
     }

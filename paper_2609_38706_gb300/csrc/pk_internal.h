@@ -29,6 +29,7 @@ struct pk_ctx {
     pk_entry *table;
     unsigned long long *counter_dev;  // number of entries in the table
     unsigned long long epoch;         // last store call number
+    unsigned long long *stamps;       // budget mode: last-use stamp per entry (pk_attach_stamps), else NULL
     uint32_t pad_kw[64];              // K_t + W_t of a chunk's final (padding-only) block, C % 16 == 0
 };
 
@@ -65,6 +66,11 @@ cudaError_t pk_launch_content_digest(const uint8_t *bytes, uint64_t n_bytes, uin
 cudaError_t pk_launch_compare_pages(const uint32_t *slots, const uint8_t *pages, const uint8_t *ref_pages, uint64_t n,
                                     uint64_t n_ref, uint64_t page_bytes, int32_t *verdict, unsigned long long *counts,
                                     int32_t *status, cudaStream_t s);
+uint64_t pk_evict_scratch_bytes_impl(uint64_t capacity);
+cudaError_t pk_launch_evict(const pk_ctx *ctx, uint64_t budget, uint64_t keep, void *scratch, uint32_t *evicted,
+                            uint64_t evicted_cap, unsigned long long *n_evicted, int32_t *status, cudaStream_t s);
+cudaError_t pk_launch_key_strings(const uint8_t *keys, uint64_t n, const uint8_t *prefix, uint32_t plen,
+                                  uint32_t width, uint8_t *out, cudaStream_t s);
 cudaError_t pk_launch_lookup_store(const pk_ctx *ctx, unsigned long long epoch, const uint8_t *keys,
                                    const uint32_t *new_slots, const int64_t *key_off, uint32_t R,
                                    uint64_t key_capacity, int32_t *hit_chunks, uint32_t *slots, int32_t *result,

@@ -379,12 +379,17 @@ __device__ __forceinline__ void bid(pk_entry *ent, uint32_t me, uint32_t my_slot
 // the table when the call started (inserted by an earlier call: epoch set
 // and not this call's), else PK_NO_SLOT; a key that may not be inserted
 // (!may_claim) ends with PK_ERR_ARG and leaves the table untouched.
+// stamps (budget mode, else NULL): the last-use stamp (epoch << 32) | e of
+// the key's entry is raised to this entry's when the key was in the table at
+// the start of the call, or is inserted by it with a valid slot.
 template <bool kFused>
 __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cur, const uint4 &key, uint32_t me,
                                            uint32_t my_slot, unsigned long long epoch, bool fast,
                                            unsigned long long *counter, uint64_t capacity, bool may_claim,
-                                           int32_t &res, uint32_t &out, uint32_t &lslot) {
+                                           unsigned long long *stamps, int32_t &res, uint32_t &out,
+                                           uint32_t &lslot) {
     uint4 *kp = reinterpret_cast<uint4 *>(ent->k);
+    const unsigned long long my_stamp = (epoch << 32) | (unsigned long long)(uint32_t)~me;
     lslot = PK_NO_SLOT;
 #pragma unroll 1
     for (int pass = 0; pass < 2; ++pass) {
@@ -403,10 +408,12 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
                 if (kFused) lslot = sl;
                 res = (!kFused || may_claim) ? PK_STORE_PRESENT : PK_ERR_ARG;
                 out = (!kFused || may_claim) ? sl : PK_NO_SLOT;
+                if (stamps) atomicMax(stamps + pos, my_stamp);
             } else if (!kFused || may_claim) {  // claimed during this call
                 bid(ent, me, my_slot);
                 res = PK_STORE_PENDING;
                 out = (uint32_t)pos;
+                if (stamps) atomicMax(stamps + pos, my_stamp);
             } else {
                 res = PK_ERR_ARG;
                 out = PK_NO_SLOT;
@@ -430,6 +437,7 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
         if (is_zero(old)) {  // claimed
             *(volatile unsigned long long *)&ent->epoch = epoch;
             bid(ent, me, my_slot);
+            if (stamps) atomicMax(stamps + pos, my_stamp);
             res = PK_STORE_PENDING;
             out = (uint32_t)pos;
             if (fast) return kClaimedHere;  // counted once per block at the end
@@ -457,6 +465,7 @@ struct ClaimCtx {
     unsigned long long *counter;
     unsigned long long epoch;
     bool fast;
+    unsigned long long *stamps;  // budget mode: last-use stamp per entry, else NULL
 };
 
 // Insert-if-absent: one round over the undecided keys P of the warp.
@@ -513,7 +522,7 @@ __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, Probe
     if (decider) {
         const uint64_t epos = wb + (uint32_t)cand;
         const Examine x = examine<kFused>(c.table + epos, epos, cv, k, ~(uint32_t)we, wslot, c.epoch, c.fast,
-                                          c.counter, c.capacity, wmay, dres, dout, dls);
+                                          c.counter, c.capacity, wmay, c.stamps, dres, dout, dls);
         if (x == kClaimedHere) ++claims;
         if (x == kAdvance) {  // lost the entry to a different key: continue after it
             dadv = true;
@@ -616,7 +625,7 @@ __device__ __forceinline__ void count_claims(unsigned long long *block_claims, u
 // consecutive entries.
 __global__ void __launch_bounds__(256, 4)
 k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
-              unsigned long long *counter, unsigned long long epoch, const uint8_t *keys,
+              unsigned long long *counter, unsigned long long epoch, unsigned long long *stamps, const uint8_t *keys,
               const uint32_t *slots, uint64_t n, const int64_t *key_off,
               const int32_t *hit, uint32_t R, int32_t *result,
               uint32_t *slot_out, int32_t *status) {
@@ -631,7 +640,7 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
     unsigned long long cnt = 0;
     if (lane == 0) cnt = ld_volatile_u64(counter);
     const bool fast = __shfl_sync(kFull, cnt, 0) + n < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast};
+    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast, stamps};
     int32_t res = PK_STORE_SKIPPED;
     uint32_t out = PK_NO_SLOT;
     ProbeKey s;
@@ -655,9 +664,9 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
 // Range mode for many short requests: one warp per request, no search.
 // Writes every entry of [key_off[r], key_off[r+1]); entries past key_off[R]
 // are marked by the finalize kernel.
-__global__ void __launch_bounds__(256, 4)
+__global__ void __launch_bounds__(256, 3)
 k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
-                  unsigned long long *counter, unsigned long long epoch, const uint8_t *keys,
+                  unsigned long long *counter, unsigned long long epoch, unsigned long long *stamps, const uint8_t *keys,
                   const uint32_t *slots, uint64_t n, const int64_t *key_off,
                   const int32_t *hit, uint32_t R, int32_t *result,
                   uint32_t *slot_out, int32_t *status) {
@@ -678,7 +687,7 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
     unsigned long long cnt = 0;
     if (lane == 0) cnt = ld_volatile_u64(counter);
     const bool fast = __shfl_sync(kFull, cnt, 0) + n < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast};
+    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast, stamps};
     uint32_t claims = 0;
     for (int64_t x = a + lane; x < first && x < b; x += 32) {  // below h_r: not stored
         result[x] = PK_STORE_SKIPPED;
@@ -754,7 +763,7 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
 // One warp per request, refilled from a register buffer as k_lookup_req.
 __global__ void __launch_bounds__(256, 3)
 k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
-                   unsigned long long *counter, unsigned long long epoch, const uint8_t *keys,
+                   unsigned long long *counter, unsigned long long epoch, unsigned long long *stamps, const uint8_t *keys,
                    const uint32_t *new_slots, const int64_t *key_off, uint32_t R,
                    uint64_t key_capacity, uint32_t *slots, int32_t *hit,
                    int32_t *result, uint32_t *slot_out, int32_t *status) {
@@ -773,7 +782,7 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
     unsigned long long cnt = 0;
     if (lane == 0) cnt = ld_volatile_u64(counter);
     const bool fast = __shfl_sync(kFull, cnt, 0) + key_capacity < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast};
+    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast, stamps};
     uint32_t claims = 0;
     uint32_t first_miss = 0xffffffffu;  // lowest miss index (relative to a) seen by this lane
     int64_t arg_hit = -1;               // highest index of a hit whose slot was PK_NO_SLOT
@@ -850,7 +859,7 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
 // then finds h_r and relabels.
 __global__ void __launch_bounds__(256)
 k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity, unsigned long long *counter,
-               unsigned long long epoch, const uint8_t *keys, const uint32_t *new_slots,
+               unsigned long long epoch, unsigned long long *stamps, const uint8_t *keys, const uint32_t *new_slots,
                const int64_t *key_off, uint32_t R, uint64_t key_capacity, uint32_t *slots,
                int32_t *result, uint32_t *slot_out, int32_t *status) {
     __shared__ unsigned long long block_claims;
@@ -864,7 +873,7 @@ k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capa
     unsigned long long cnt = 0;
     if (lane == 0) cnt = ld_volatile_u64(counter);
     const bool fast = __shfl_sync(kFull, cnt, 0) + key_capacity < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast};
+    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast, stamps};
     int32_t res = PK_STORE_SKIPPED;
     uint32_t out = PK_NO_SLOT, lslot = PK_NO_SLOT;
     ProbeKey s;
@@ -1013,7 +1022,7 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
     unsigned long long cnt = 0;
     if (lane == 0) cnt = ld_volatile_u64(&sc->count);
     const bool fast = __shfl_sync(kFull, cnt, 0) + n < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, &sc->count, epoch, fast};
+    const ClaimCtx c{table, mask, max_probe, capacity, &sc->count, epoch, fast, nullptr};
     int32_t res = PK_STORE_SKIPPED;
     uint32_t out = PK_NO_SLOT;
     ProbeKey s;
@@ -1092,11 +1101,11 @@ cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const u
     cudaError_t e;
     if (key_off && R > 0 && per_request(R, n)) {
         e = pk_launch(k_store_claim_req, grid_for(32ull * R, 256), 256, s, ctx->table, mask, ctx->max_probe,
-                      ctx->capacity, ctx->counter_dev, epoch, keys, slots, n, key_off, hit_chunks, R, result,
+                      ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, slots, n, key_off, hit_chunks, R, result,
                       slot_out, status);
     } else {
         e = pk_launch(k_store_claim, grid_for(n, 256), 256, s, ctx->table, mask, ctx->max_probe, ctx->capacity,
-                      ctx->counter_dev, epoch, keys, slots, n, key_off, hit_chunks, R, result, slot_out, status);
+                      ctx->counter_dev, epoch, ctx->stamps, keys, slots, n, key_off, hit_chunks, R, result, slot_out, status);
     }
     if (e == cudaSuccess)
         e = pk_launch(k_store_finalize, grid_for(n, 256), 256, s, (const pk_entry *)ctx->table, n, key_off, R, result,
@@ -1113,13 +1122,13 @@ cudaError_t pk_launch_lookup_store(const pk_ctx *ctx, unsigned long long epoch, 
     cudaError_t e;
     if (per_request(R, key_capacity)) {
         e = pk_launch(k_lookup_store_req, grid_for(32ull * R, 256), 256, s, ctx->table, mask, ctx->max_probe,
-                      ctx->capacity, ctx->counter_dev, epoch, keys, new_slots, key_off, R, key_capacity, slots,
+                      ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, new_slots, key_off, R, key_capacity, slots,
                       hit_chunks, result, slot_out, status);
     } else {
         e = key_capacity == 0
                 ? cudaSuccess
                 : pk_launch(k_lookup_store, grid_for(key_capacity, 256), 256, s, ctx->table, mask, ctx->max_probe,
-                            ctx->capacity, ctx->counter_dev, epoch, keys, new_slots, key_off, R, key_capacity, slots,
+                            ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, new_slots, key_off, R, key_capacity, slots,
                             result, slot_out, status);
         if (e == cudaSuccess)
             e = pk_launch(k_lookup_store_tail, grid_for(32ull * R, 256), 256, s, key_off, R, key_capacity,

@@ -27,6 +27,7 @@ PK_ERR_PROBE_LIMIT = -6
 PK_ERR_RESERVED_KEY = -7
 PK_ERR_CUDA = -8
 PK_ERR_TOO_LARGE = -9
+PK_ERR_TIMEOUT = -10
 PK_PAGE_ABSENT, PK_PAGE_EQUAL, PK_PAGE_DIFFERS = 0, 1, 2
 PK_NOALLOC_MAX_ENTRIES = 1 << 18
 PK_STORE_SKIPPED = 0
@@ -35,6 +36,8 @@ PK_STORE_PRESENT = 2
 PK_NO_SLOT = 0xFFFFFFFF
 PK_KEY_BYTES = 32
 PK_ENTRY_BYTES = 32
+PK_KEY_STRING_CHARS = 22
+PK_KEY_STRING_MAX_WIDTH = 256
 REGISTRY_V1 = ("model_id", "weight_precision", "weight_version", "adapter_id", "kv_format", "salt")
 
 
@@ -100,6 +103,13 @@ def lib() -> ctypes.CDLL:
             "pk_tensor_identity": (ctypes.c_int, [ctypes.POINTER(pk_bytes), ctypes.POINTER(pk_bytes), _VP, _U32,
                                                   _U64, _VP, _VP]),
             "pk_adapter_identity": (ctypes.c_int, [_VP, _U32, ctypes.POINTER(pk_bytes), _U32, _VP]),
+            "pk_stamps_bytes": (ctypes.c_size_t, [_U32]),
+            "pk_attach_stamps": (ctypes.c_int, [_VP, _VP, ctypes.c_size_t, _VP]),
+            "pk_evict_scratch_bytes": (ctypes.c_size_t, [_U32]),
+            "pk_evict": (ctypes.c_int, [_VP, _U64, _U64, _VP, ctypes.c_size_t, _VP, _U64, _VP, _VP, _VP]),
+            "pk_key_string": (ctypes.c_int, [_VP, _VP]),
+            "pk_model_tag": (ctypes.c_int, [ctypes.POINTER(pk_descriptor), _VP]),
+            "pk_key_strings": (ctypes.c_int, [_VP, _U64, _VP, _U32, _U32, _VP, _VP]),
             "pk_table_save": (ctypes.c_int, [_VP, _VP, ctypes.c_size_t, _VP]),
             "pk_table_load": (ctypes.c_int, [_VP, _VP, ctypes.c_size_t, _VP]),
             "pk_strerror": (ctypes.c_char_p, [ctypes.c_int]),
@@ -358,6 +368,56 @@ def pk_adapter_identity(tensor_ids, config) -> bytes:
     out = (ctypes.c_uint8 * 32)()
     _check(lib().pk_adapter_identity(ids.ctypes.data, len(tensor_ids), arr, len(keep), out), "pk_adapter_identity")
     return bytes(out)
+
+
+def pk_stamps_bytes(capacity_log2: int) -> int:
+    return int(lib().pk_stamps_bytes(capacity_log2))
+
+
+def pk_attach_stamps(ctx: int, stamps: Optional[torch.Tensor], stream=None) -> None:
+    """Budget mode on (stamps: device buffer of pk_stamps_bytes, zeroed here) or off (None)."""
+    nbytes = 0 if stamps is None else stamps.numel() * stamps.element_size()
+    _check(lib().pk_attach_stamps(ctx, _p(stamps), nbytes, _s(stream)), "pk_attach_stamps")
+
+
+def pk_evict_scratch_bytes(capacity_log2: int) -> int:
+    return int(lib().pk_evict_scratch_bytes(capacity_log2))
+
+
+def pk_evict(ctx: int, budget: int, keep: int, scratch: torch.Tensor, evicted: Optional[torch.Tensor],
+             n_evicted: Optional[torch.Tensor], status: torch.Tensor, stream=None) -> None:
+    """evicted: uint32/int32 [cap] device (or None); n_evicted: int64[1] device (or None)."""
+    _check(lib().pk_evict(ctx, budget, keep, _p(scratch), scratch.numel(), _p(evicted),
+                          0 if evicted is None else evicted.numel(), _p(n_evicted), _p(status), _s(stream)),
+           "pk_evict")
+
+
+def pk_key_string(key16: bytes) -> str:
+    """The 22 base64 characters of a 16-byte key prefix (host)."""
+    if len(bytes(key16)) != 16:
+        raise PKError(PK_ERR_ARG, "pk_key_string")
+    k = (ctypes.c_uint8 * 16).from_buffer_copy(bytes(key16))
+    out = (ctypes.c_char * 22)()
+    _check(lib().pk_key_string(k, out), "pk_key_string")
+    return out.raw.decode("ascii")
+
+
+def pk_model_tag(desc) -> str:
+    """The 22-character hash of the model identity and worker provenance (host)."""
+    d = _descs([desc]) if isinstance(desc, Mapping) else _descs(desc)
+    out = (ctypes.c_char * 22)()
+    _check(lib().pk_model_tag(d.array, out), "pk_model_tag")
+    return out.raw.decode("ascii")
+
+
+def pk_key_strings(keys: torch.Tensor, prefix: bytes, width: int, out: torch.Tensor, n: Optional[int] = None,
+                   stream=None) -> None:
+    """out (uint8 [n, width], device): row i = prefix || base64 of keys[i, :16] || zero fill."""
+    n = keys.shape[0] if n is None else n
+    pre = bytes(prefix)
+    buf = ctypes.create_string_buffer(pre, max(len(pre), 1))
+    _check(lib().pk_key_strings(_p(keys), n, ctypes.cast(buf, ctypes.c_void_p), len(pre), width, _p(out),
+                                _s(stream)), "pk_key_strings")
 
 
 def pk_table_save(ctx: int, dst: torch.Tensor, stream=None) -> None:

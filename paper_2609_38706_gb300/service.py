@@ -159,6 +159,26 @@ class KeyTable:
                            self.stream)
         return hit, slots, result, slot_out
 
+    # -- budget mode (eviction under a fixed budget) -------------------------
+    def attach_stamps(self) -> torch.Tensor:
+        """Turn budget mode on: a zeroed last-use stamp per entry, and the
+        scratch and output buffers of evict()."""
+        cap = 1 << self.capacity_log2
+        self.stamps = torch.empty(pk.pk_stamps_bytes(self.capacity_log2) // 8, dtype=torch.int64, device=self.device)
+        pk.pk_attach_stamps(self.ctx, self.stamps, self.stream)
+        self.evict_scratch = torch.empty(pk.pk_evict_scratch_bytes(self.capacity_log2), dtype=torch.uint8,
+                                         device=self.device)
+        self.evicted = torch.empty(cap, dtype=torch.int32, device=self.device)
+        self.n_evicted = torch.zeros(1, dtype=torch.int64, device=self.device)
+        return self.stamps
+
+    def evict(self, budget: int, keep: int):
+        """Enqueue pk_evict; returns (evicted slots buffer, count tensor),
+        valid up to the count once the stream has run."""
+        pk.pk_evict(self.ctx, budget, keep, self.evict_scratch, self.evicted, self.n_evicted, self.status,
+                    self.stream)
+        return self.evicted, self.n_evicted
+
     def seed(self, seed_keys, filler, target_entries: int) -> int:
         """Pre-fill: seed keys in order (slot = list index), then filler keys
         (continuing the index) until the table holds target_entries entries."""

@@ -35,3 +35,17 @@ def load_golden_sha256():
 @pytest.fixture(scope="session")
 def golden_sha256():
     return load_golden_sha256()
+
+
+def load_golden_base64():
+    """Parse tests/golden/rfc4648_base64_vectors.txt -> [(input bytes, encoding str)]."""
+    out = []
+    path = os.path.join(ROOT, "tests", "golden", "rfc4648_base64_vectors.txt")
+    with open(path) as f:
+        for line in f:
+            line = line.rstrip("\n")
+            if not line or line.startswith("#"):
+                continue
+            a, b = line.split("\t")
+            out.append((b"" if a == "<empty>" else a.encode(), "" if b == "<empty>" else b))
+    return out

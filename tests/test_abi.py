@@ -189,3 +189,34 @@ def test_null_context_rejected(pk):
     assert L.pk_lookup_store(None, None, None, None, 0, 0, None, None, None, None, None, None) == pk.PK_ERR_ARG
     assert L.pk_derive_keys(None, None, 0, None, 0, None, None, 0, None, None, 0, None, None) == pk.PK_ERR_ARG
     assert L.pk_destroy(None) == pk.PK_ERR_ARG
+
+
+def test_key_string_and_model_tag_match_oracle(pk):
+    rng = np.random.default_rng(21)
+    for _ in range(300):
+        p = rng.integers(0, 256, 16, dtype=np.uint8).tobytes()
+        assert pk.pk_key_string(p) == O.key_string(p)
+    for _ in range(50):
+        d = _rand_desc(rng)
+        try:
+            want = O.model_tag(d)
+        except O.OracleError as e:
+            with pytest.raises(pk.PKError) as ei:
+                pk.pk_model_tag(d)
+            assert ei.value.code == e.code
+            continue
+        assert pk.pk_model_tag(d) == want
+
+
+def test_key_strings_host_errors_before_any_cuda_call(pk):
+    L = pk.lib()
+    fake = ctypes.c_void_p(1 << 40)  # never dereferenced: every case fails its host check
+    assert L.pk_key_strings(fake, 4, None, 0, 21, fake, None) == pk.PK_ERR_ARG           # width < 22
+    assert L.pk_key_strings(fake, 4, None, 0, 257, fake, None) == pk.PK_ERR_ARG          # width > max
+    assert L.pk_key_strings(fake, 4, b"abc", 3, 24, fake, None) == pk.PK_ERR_ARG         # prefix + 22 > width
+    assert L.pk_key_strings(fake, 4, None, 2, 64, fake, None) == pk.PK_ERR_ARG           # prefix NULL
+    assert L.pk_key_strings(None, 4, None, 0, 22, fake, None) == pk.PK_ERR_ARG           # keys NULL
+    assert L.pk_key_strings(fake, 4, None, 0, 22, None, None) == pk.PK_ERR_ARG           # out NULL
+    assert L.pk_key_strings(ctypes.c_void_p((1 << 40) + 8), 4, None, 0, 22, fake, None) == pk.PK_ERR_ARG
+    assert L.pk_key_strings(fake, 4, None, 0, 22, ctypes.c_void_p((1 << 40) + 4), None) == pk.PK_ERR_ARG
+    assert L.pk_key_strings(None, 0, None, 0, 22, None, None) == pk.PK_OK                # empty batch
