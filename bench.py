@@ -523,6 +523,138 @@ def main():
     cmp_gbs = cmp_bytes / (float(np.mean(cmp_ms)) / 1e3) / 1e9
     del ref_pages, pages
 
+    # Connector key strings (pk_key_strings): the step's keys as 150-byte rows (prefix, 22 base64
+    # characters, zero fill), and 16M random keys (2.4 GB of rows) for the HBM roofline.
+    ks_width = 150
+    ks_prefix = ("vllm@" + pk.pk_model_tag(wl.descriptors[0]) + "@1@0@").encode()
+
+    def key_strings_us(keys, n, reps=8):
+        rows = torch.empty((n, ks_width), dtype=torch.uint8, device=dev)
+        times = []
+        for it in range(reps + 3):
+            flush.fill_(1)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            pk.pk_key_strings(keys, ks_prefix, ks_width, rows, n=n)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if it >= 3:
+                times.append(e0.elapsed_time(e1) * 1e3)
+        del rows
+        return float(np.mean(times))
+    ks_step_us = key_strings_us(keys_d, n_keys)
+    n_big = 16 << 20
+    big_keys = torch.randint(0, 256, (n_big, 32), dtype=torch.uint8, device=dev, generator=gen)
+    ks_big_us = key_strings_us(big_keys, n_big, reps=5)
+    del big_keys
+    ks_bytes = n_big * (16 + ks_width)
+    ks_gbs = ks_bytes / (ks_big_us * 1e-6) / 1e9
+    line["key_strings"] = {
+        "step_keys": n_keys, "step_us": ks_step_us, "width": ks_width, "prefix_bytes": len(ks_prefix),
+        "roofline": {"bound": "hbm", "kernel": "pk_key_strings", "keys": n_big, "us": ks_big_us,
+                     "achieved": ks_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": ks_gbs / peaks["hbm_gbs"],
+                     "bytes_basis": f"16 B key prefix read + {ks_width} B row written per key",
+                     "peak_source": peaks["source"]}}
+
+    # Eviction under a fixed budget (pk_evict).  (1) The kernel on a 2^22-entry table holding 2M entries
+    # (stamps from one list-mode store), evicting to 1M: restored and L2-flushed before each repetition.
+    # (2) The call within the budget (returns at once).  (3) The thrashing of Sec. 6.5 on the key path:
+    # one prompt pool served under D adapters in turn, budget about one copy of the pool, evicting after
+    # every step; bound keys (one copy per adapter) against unbound keys (one copy in all).
+    ev_log2, ev_n = 22, 2 << 20
+    kt_ev = KeyTable(16, ev_log2, device=dev)
+    kt_ev.attach_stamps()
+    ev_keys = torch.randint(0, 256, (ev_n, 32), dtype=torch.uint8, device=dev, generator=gen)
+    ev_keys[:, 0] |= 1
+    kt_ev.store(ev_keys, torch.arange(ev_n, dtype=torch.int32, device=dev))
+    del ev_keys
+    torch.cuda.synchronize()
+    if kt_ev.take_status() != 0:
+        raise RuntimeError("eviction table fill")
+    ev_entries = kt_ev.entries()
+    ev_snap, ev_stamps = kt_ev.save(), kt_ev.stamps.clone()
+
+    def evict_us(budget, keep, reps):
+        times, n_out = [], 0
+        for it in range(reps + 2):
+            kt_ev.load(ev_snap)
+            kt_ev.stamps.copy_(ev_stamps)
+            flush.fill_(1)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            _, n_ev = kt_ev.evict(budget, keep)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if it >= 2:
+                times.append(e0.elapsed_time(e1) * 1e3)
+            n_out = int(n_ev.item())
+        if kt_ev.take_status() != 0:
+            raise RuntimeError("evict status")
+        return float(np.mean(times)), n_out
+    ev_keep = ev_entries // 2
+    ev_us, ev_removed = evict_us(ev_entries - 1, ev_keep, 5)
+    if ev_removed != ev_entries - ev_keep or kt_ev.entries() != ev_keep:
+        raise RuntimeError("eviction count")
+    idle_us, idle_removed = evict_us(ev_entries, ev_keep, 10)
+    kt_ev.close()
+    del kt_ev, ev_snap, ev_stamps
+    # bytes: the gather reads one 32 B entry sector per table entry and 8 B of stamp per entry held; the
+    # compaction rewrites the removed entries (32 B + 8 B of stamp each)
+    ev_bytes = (1 << ev_log2) * 32 + ev_entries * 8 + ev_removed * 40
+    thrash = []
+    for D in (1, 2, 4):
+        for bound in ((True,) if D == 1 else (True, False)):
+            es = W.eviction_stream(D)
+            kts = KeyTable(es.chunk_tokens, 14, device=dev)
+            kts.attach_stamps()
+            dg = kts.digests(es.descriptors)
+            pool_d = torch.from_numpy(es.pool).to(dev)
+            Rs, kch = es.requests_per_step, es.pool.shape[1] // es.chunk_tokens
+            tok_off_s = torch.arange(Rs + 1, dtype=torch.int64, device=dev) * es.pool.shape[1]
+            key_off_s = torch.empty(Rs + 1, dtype=torch.int64, device=dev)
+            keys_s = torch.empty((Rs * kch, 32), dtype=torch.uint8, device=dev)
+            hit_s = torch.empty(Rs, dtype=torch.int32, device=dev)
+            outs = torch.empty((3, Rs * kch), dtype=torch.int32, device=dev)
+            cyc = es.steps_per_cycle()
+            hits = chunks = evicted = 0
+            st_us = []
+            for s in range(3 * cyc):
+                bt = es.step(s, bound)
+                first = (s * Rs) % es.P
+                toks = pool_d[first:first + Rs].reshape(-1)
+                didx = torch.full((Rs,), int(bt.desc_idx[0]), dtype=torch.int32, device=dev)
+                slots_new = torch.arange(Rs * kch, dtype=torch.int32, device=dev) + s * Rs * kch
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                pk.pk_derive_keys(kts.ctx, toks, tok_off_s, didx, dg, key_off_s, keys_s, kts.status)
+                pk.pk_lookup_store(kts.ctx, keys_s, slots_new, key_off_s, hit_s, outs[0], outs[1], outs[2],
+                                   kts.status)
+                _, n_ev = kts.evict(es.budget, es.budget)
+                e1.record(stream)
+                torch.cuda.synchronize()
+                if s >= cyc:  # after the first cycle
+                    st_us.append(e0.elapsed_time(e1) * 1e3)
+                    hits += int(hit_s.sum().item())
+                    chunks += Rs * kch
+                    evicted += int(n_ev.item())
+            if kts.take_status() != 0:
+                raise RuntimeError("thrash status")
+            thrash.append({"D": D, "bound": bound, "hit_rate": hits / chunks, "step_us": float(np.mean(st_us)),
+                           "evicted_per_step": evicted / len(st_us), "working_set_chunks": (D if bound else 1)
+                           * es.P * kch, "budget_chunks": es.budget})
+            kts.close()
+    line["eviction"] = {
+        "evict_us": ev_us, "table_entries": ev_entries, "removed": ev_removed, "capacity": 1 << ev_log2,
+        "within_budget_us": idle_us,
+        "achieved_GBps": ev_bytes / (ev_us * 1e-6) / 1e9, "peak_GBps": peaks["hbm_gbs"],
+        "frac": ev_bytes / (ev_us * 1e-6) / 1e9 / peaks["hbm_gbs"],
+        "bytes_basis": "32 B entry sector per table entry + 8 B stamp per entry held + 40 B per removed entry",
+        "thrash": thrash,
+        "thrash_setup": "512 prompts x 8 chunks of 256 tokens, 64 requests per step, prompt i % 512 under "
+                        "adapter (i // 512) % D, budget 4608 entries (1.125 copies), evict after each step; "
+                        "hit rate and step time (derive + lookup-and-store + evict) over cycles 2-3",
+        "paper": "vLLM, bound: TTFT 0.024 -> 0.065 s, 42 -> 15 req/s once capacity is exceeded; unbound flat"}
+
     # Content identity (pk_content_digest, the SHA-256 tree): a 40 MB adapter as 16 tensors, and a 1 GiB
     # checkpoint buffer; random bytes generated on the device.
     def content_us(sizes, reps=5):

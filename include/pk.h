@@ -341,11 +341,11 @@ int pk_key_strings(const uint8_t *keys_dev, uint64_t n, const char *prefix, uint
  * nothing.  Entries stored before the stamps were attached (or before a
  * pk_table_load) have stamp 0.
  *   pk_stamps_bytes:  bytes of the stamp array (8 per entry; 0 if out of range).
- *   pk_attach_stamps: enable budget mode with stamps_dev (8-byte aligned,
+ *   pk_attach_stamps: enable budget mode with stamps_dev (16-byte aligned,
  *                     >= pk_stamps_bytes) and zero it on `stream`; NULL
  *                     detaches.
- *   pk_evict_scratch_bytes: device scratch pk_evict needs (about 8.2 bytes
- *                     per entry plus 8.5 KiB).
+ *   pk_evict_scratch_bytes: device scratch pk_evict needs (about 13.3
+ *                     bytes per entry plus 8.5 KiB).
  *   pk_evict (device): when the table holds more than `budget` entries,
  *                     remove every entry whose stamp is at most v, the
  *                     (keep+1)-th largest stamp: the least recently used

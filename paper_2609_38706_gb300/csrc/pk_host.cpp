@@ -370,7 +370,7 @@ int pk_attach_stamps(pk_ctx *ctx, uint64_t *stamps_dev, size_t stamps_bytes, pk_
         ctx->stamps = nullptr;
         return PK_OK;
     }
-    if (!aligned(stamps_dev, 8) || stamps_bytes < pk_stamps_bytes(ctx->capacity_log2)) return PK_ERR_ARG;
+    if (!aligned16(stamps_dev) || stamps_bytes < pk_stamps_bytes(ctx->capacity_log2)) return PK_ERR_ARG;
     if (cudaMemsetAsync(stamps_dev, 0, pk_stamps_bytes(ctx->capacity_log2), reinterpret_cast<cudaStream_t>(stream)) !=
         cudaSuccess)
         return PK_ERR_CUDA;

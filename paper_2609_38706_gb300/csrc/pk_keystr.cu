@@ -8,12 +8,16 @@
 // where the prefix (the connector's fixed fields and the model tag) is the
 // same for every row.
 //
-// The rows of 256 keys form one contiguous tile of the output (256 * width is
-// a multiple of 16), written as coalesced 16-byte stores: each thread first
-// encodes the 22 characters of one key into shared memory, then the block
-// assembles the tile 16 bytes per thread from the prefix, the characters and
-// zeros.  Output bytes dominate the traffic (width against 16 key bytes read
-// per row), so the kernel is bound by HBM writes.
+// Output bytes dominate the traffic (the row width against 16 key bytes read
+// per row), so the kernel is built to write at HBM speed: a persistent grid,
+// each CTA holding two tiles of 256 rows in shared memory, laid out exactly
+// as in the output (256 * width bytes, a multiple of 16) and filled once with
+// the prefix and zeros.  Per tile only the 22 characters of each row change:
+// every thread encodes its key into its row, then one thread hands the whole
+// tile to the TMA engine as a single bulk store (cp.async.bulk, shared to
+// global).  The two tiles alternate, so encoding the next tile overlaps the
+// store of the previous one, and each thread's next key is loaded a tile
+// ahead.
 #include <cuda_runtime.h>
 
 #include "pk_device.cuh"
@@ -21,7 +25,7 @@
 
 namespace {
 
-constexpr uint32_t kRows = 256;  // keys (rows) per block; also threads per block
+constexpr uint32_t kRows = 256;  // rows per tile; one thread per row
 constexpr uint32_t kChars = PK_KEY_STRING_CHARS;
 
 struct KeyStrArgs {
@@ -36,58 +40,73 @@ __device__ __forceinline__ uint8_t b64_char(uint32_t v) {  // v < 64
 
 __device__ __forceinline__ uint32_t bswap32(uint32_t x) { return __byte_perm(x, 0, 0x0123); }
 
-__global__ void __launch_bounds__(kRows) k_key_strings(const uint8_t *keys, uint64_t n, KeyStrArgs a, uint8_t *out) {
-    __shared__ uint8_t pre[PK_KEY_STRING_MAX_WIDTH];
-    __shared__ uint8_t chars[kRows * kChars];
-    pk::pdl_wait(keys, out);
-    const uint32_t t = threadIdx.x;
-    const uint64_t row0 = (uint64_t)blockIdx.x * kRows;
-    const uint32_t rows = (uint32_t)min((uint64_t)kRows, n - row0);
-    for (uint32_t j = t; j < a.plen; j += kRows) pre[j] = a.prefix[j];
-    if (t < rows) {
-        // The 16 bytes as a 128-bit big-endian integer (hi, lo); character q
-        // is bits [6q, 6q + 6) counted from the most significant bit.
-        const uint4 k = __ldcg(reinterpret_cast<const uint4 *>(keys + 32 * (row0 + t)));
-        const uint64_t hi = ((uint64_t)bswap32(k.x) << 32) | bswap32(k.y);
-        const uint64_t lo = ((uint64_t)bswap32(k.z) << 32) | bswap32(k.w);
-        uint8_t *c = chars + t * kChars;
+// Bulk copy of `bytes` (a multiple of 16) from shared to global memory,
+// tracked in this thread's bulk group.
+__device__ __forceinline__ void bulk_store(void *gdst, const void *ssrc, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
+                 :
+                 : "l"(gdst), "r"((uint32_t)__cvta_generic_to_shared(ssrc)), "r"(bytes)
+                 : "memory");
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// At most one bulk group of this thread still reading shared memory.
+__device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+// Every bulk group of this thread complete.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// Shared-memory writes of this thread visible to the TMA engine (async proxy).
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__device__ __forceinline__ void encode_row(const uint4 &k, uint8_t *c) {
+    // The 16 bytes as a 128-bit big-endian integer (hi, lo); character q is
+    // bits [6q, 6q + 6) counted from the most significant bit.
+    const uint64_t hi = ((uint64_t)bswap32(k.x) << 32) | bswap32(k.y);
+    const uint64_t lo = ((uint64_t)bswap32(k.z) << 32) | bswap32(k.w);
 #pragma unroll
-        for (uint32_t q = 0; q < kChars; ++q) {
-            const uint32_t s = 6 * q;  // <= 126
-            const uint64_t top = s == 0 ? hi : s < 64 ? (hi << s) | (lo >> (64 - s)) : lo << (s - 64);
-            c[q] = b64_char((uint32_t)(top >> 58));
-        }
+    for (uint32_t q = 0; q < kChars; ++q) {
+        const uint32_t s = 6 * q;  // <= 126
+        const uint64_t top = s == 0 ? hi : s < 64 ? (hi << s) | (lo >> (64 - s)) : lo << (s - 64);
+        c[q] = b64_char((uint32_t)(top >> 58));
     }
+}
+
+__global__ void __launch_bounds__(kRows) k_key_strings(const uint8_t *keys, uint64_t n, KeyStrArgs a, uint8_t *out) {
+    extern __shared__ __align__(128) uint8_t sm[];  // two tiles of kRows * width bytes
+    const uint32_t t = threadIdx.x;
+    const uint32_t tile_bytes = kRows * a.width;
+    // Both tiles: zeros, then the prefix at the start of every row.
+    uint4 *sm4 = reinterpret_cast<uint4 *>(sm);
+    for (uint32_t i = t; i < 2 * tile_bytes / 16; i += kRows) sm4[i] = make_uint4(0, 0, 0, 0);
     __syncthreads();
-    // Tile bytes [0, rows * width); unit u = bytes [16u, 16u + 16).
-    const uint64_t bytes = (uint64_t)rows * a.width;
-    uint8_t *dst = out + row0 * a.width;
-    for (uint64_t u = t; 16 * u < bytes; u += kRows) {
-        uint64_t o = 16 * u;
-        uint32_t r = (uint32_t)(o / a.width), col = (uint32_t)(o - (uint64_t)r * a.width);
-        uint32_t w[4] = {0, 0, 0, 0};
-        const uint32_t nb = (uint32_t)min((uint64_t)16, bytes - o);
-#pragma unroll
-        for (uint32_t b = 0; b < 16; ++b) {
-            if (b < nb) {
-                const uint32_t v =
-                    col < a.plen ? pre[col] : col < a.plen + kChars ? chars[r * kChars + col - a.plen] : 0u;
-                w[b >> 2] |= v << (8 * (b & 3));
-                if (++col == a.width) {
-                    col = 0;
-                    ++r;
-                }
-            }
-        }
-        if (nb == 16) {
-            *reinterpret_cast<uint4 *>(dst + o) = make_uint4(w[0], w[1], w[2], w[3]);
-        } else {  // the last bytes of the last tile
-#pragma unroll
-            for (uint32_t b = 0; b < 16; ++b)
-                if (b < nb) dst[o + b] = (uint8_t)(w[b >> 2] >> (8 * (b & 3)));
-        }
+    for (uint32_t j = 0; j < a.plen; ++j) {
+        sm[t * a.width + j] = a.prefix[j];
+        sm[tile_bytes + t * a.width + j] = a.prefix[j];
+    }
+    pk::pdl_wait(keys, out);
+    const uint64_t n_tiles = (n + kRows - 1) / kRows;
+    uint64_t tile = blockIdx.x;
+    uint4 k = make_uint4(0, 0, 0, 0);
+    if (tile * kRows + t < n) k = __ldcg(reinterpret_cast<const uint4 *>(keys + 32 * (tile * kRows + t)));
+    for (uint32_t it = 0; tile < n_tiles; tile += gridDim.x, ++it) {
+        uint8_t *buf = sm + (it & 1) * tile_bytes;
+        const uint64_t row0 = tile * kRows;
+        const uint32_t rows = (uint32_t)min((uint64_t)kRows, n - row0);
+        const uint64_t next = row0 + (uint64_t)gridDim.x * kRows + t;  // this thread's key of the next tile
+        uint4 k_next = make_uint4(0, 0, 0, 0);
+        if (next < n) k_next = __ldcg(reinterpret_cast<const uint4 *>(keys + 32 * next));
+        if (t == 0) bulk_wait_read_1();  // the store that last used `buf` has read it
+        __syncthreads();
+        if (t < rows) encode_row(k, buf + t * a.width + a.plen);
+        fence_proxy_async_smem();
+        __syncthreads();
+        const uint32_t bytes = rows * a.width;
+        const uint32_t b16 = bytes & ~15u;
+        uint8_t *dst = out + row0 * a.width;  // 16-byte aligned: 256 * width is a multiple of 16
+        if (t == 0 && b16) bulk_store(dst, buf, b16);
+        for (uint32_t j = b16 + t; j < bytes; j += kRows) dst[j] = buf[j];  // the last tile's final bytes
+        k = k_next;
     }
     pk::pdl_launch_dependents();
+    if (t == 0) bulk_wait_all();  // shared memory stays allocated until the TMA engine has read it
 }
 
 }  // namespace
@@ -99,6 +118,27 @@ cudaError_t pk_launch_key_strings(const uint8_t *keys, uint64_t n, const uint8_t
     a.plen = plen;
     a.width = width;
     for (uint32_t j = 0; j < PK_KEY_STRING_MAX_WIDTH; ++j) a.prefix[j] = j < plen ? prefix[j] : 0;
-    const cudaError_t e = pk_launch(k_key_strings, (unsigned)((n + kRows - 1) / kRows), kRows, s, keys, n, a, out);
+    const size_t smem = 2ull * kRows * width;  // <= 128 KiB
+    cudaError_t e = cudaFuncSetAttribute(k_key_strings, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)(2 * kRows * PK_KEY_STRING_MAX_WIDTH));
+    int dev = 0, sms = 0, per_sm = 0;
+    if (e == cudaSuccess) e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_key_strings, kRows, smem);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) per_sm = 1;
+    const uint64_t tiles = (n + kRows - 1) / kRows;
+    const uint64_t resident = (uint64_t)sms * per_sm;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(tiles < resident ? tiles : resident));
+    cfg.blockDim = dim3(kRows);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, k_key_strings, keys, n, a, out);
     return e != cudaSuccess ? e : cudaGetLastError();
 }

@@ -427,3 +427,50 @@ def omission_case(varied: str, omit: Optional[str], seed: int = 5, R: int = 12, 
         return dict(d, **{omit: fixed})
     return OmissionCase(f"vary {varied}, omit {omit}", C, batch, a, b, bound(a), bound(b),
                         kv_pages(batch, C, lambda r: a, page_bytes), kv_pages(batch, C, lambda r: b, page_bytes))
+
+
+# --------------------------------------------------------------------------
+# Eviction under a fixed budget (Sec. 6.5): one pool of prompts served under
+# D provenances (adapters) in turn, against a store whose budget holds about
+# one copy of the pool's chunks.  Bound keys give D distinct copies, so the
+# working set is D times the pool; unbound keys (every request keyed under
+# the first descriptor, the provenance dimension dropped) give one.
+# --------------------------------------------------------------------------
+@dataclass
+class EvictionStream:
+    chunk_tokens: int
+    descriptors: list
+    pool: np.ndarray          # int32[P, k * C]: the prompts
+    requests_per_step: int
+    budget: int               # entries (chunks)
+
+    @property
+    def P(self) -> int:
+        return int(self.pool.shape[0])
+
+    def steps_per_cycle(self) -> int:
+        """Steps until every prompt has been served under every provenance once."""
+        return len(self.descriptors) * self.P // self.requests_per_step
+
+    def step(self, s: int, bound: bool) -> Batch:
+        """Requests s*R .. s*R+R-1: request i is prompt i % P under provenance
+        (i // P) % D (all under provenance 0 when unbound)."""
+        R, P, D = self.requests_per_step, self.P, len(self.descriptors)
+        first = (s * R) % P
+        rows = self.pool[first:first + R]
+        variant = ((s * R) // P) % D if bound else 0
+        off = np.arange(R + 1, dtype=np.int64) * rows.shape[1]
+        return Batch(np.ascontiguousarray(rows).reshape(-1), off, np.full(R, variant, np.uint32))
+
+
+def eviction_stream(D: int, P: int = 512, k: int = 8, R: int = 64, C: int = 256, margin: float = 0.125,
+                    seed: int = 5) -> EvictionStream:
+    """P prompts of k chunks (C tokens, vocab 152064), R requests per step
+    (R divides P), D adapters; budget = (1 + margin) * P * k entries."""
+    if P % R:
+        raise ValueError("R must divide P")
+    rng = np.random.default_rng(seed)
+    version = _hex(rng, 20)
+    descs = [_desc(version=version, adapter=f"adapter-{a:02d}") for a in range(D)]
+    pool = rng.integers(0, 152064, (P, k * C), dtype=np.int64).astype(np.int32)
+    return EvictionStream(C, descs, pool, R, int((1 + margin) * P * k))

@@ -201,3 +201,48 @@ def test_workload_step_with_budget(name):
     assert triples(kt) == bt.triples()
     check_lookups(kt, bt, np.ascontiguousarray(keys.cpu().numpy()[:N]))
     kt.close()
+
+
+def test_all_stamps_equal():
+    """Every stamp 0 (stored before the stamps were attached): the (keep+1)-th
+    largest is 0 and every entry goes."""
+    from paper_2609_38706_gb300.service import KeyTable
+    rng = np.random.default_rng(10)
+    kt = KeyTable(16, 11)
+    bt = O.BudgetTable(1 << 11)
+    keys = _keys(rng, 900)
+    kt.store(torch.from_numpy(keys).cuda(), np.arange(900, dtype=np.uint32))
+    bt.table.store(keys, np.arange(900, dtype=np.uint32))
+    kt.attach_stamps()
+    run_evict(kt, bt, 500, 100)
+    assert len(bt) == 0 and kt.entries() == 0
+    assert not kt.table.any()
+    kt.close()
+
+
+def test_large_table_sampled():
+    """2^20 entries, 600k stored by two list-mode calls and a lookup-and-store,
+    evicted to 200k: removed slots compared in full, kept entries as a set,
+    lookups of a sample."""
+    from paper_2609_38706_gb300.service import KeyTable
+    rng = np.random.default_rng(11)
+    log2 = 20
+    kt = KeyTable(16, log2)
+    kt.attach_stamps()
+    bt = O.BudgetTable(1 << log2)
+    keys = _keys(rng, 600_000)
+    for a, b in ((0, 300_000), (300_000, 600_000)):
+        sl = np.arange(a, b, dtype=np.uint32)
+        kt.store(torch.from_numpy(keys[a:b]).cuda(), sl)
+        bt.store(keys[a:b], sl)
+    reuse = np.ascontiguousarray(keys[rng.permutation(600_000)[:50_000]])  # touch 50k of them again
+    off = np.arange(0, 50_001, 10, dtype=np.int64)
+    sl = np.arange(50_000, dtype=np.uint32) + 10_000_000
+    kt.lookup_store(torch.from_numpy(reuse).cuda(), torch.from_numpy(off).cuda(), sl)
+    bt.lookup_store(reuse, off, sl)
+    torch.cuda.synchronize()
+    kt.check("lookup_store")
+    run_evict(kt, bt, 500_000, 200_000)
+    assert triples(kt) == bt.triples()
+    check_lookups(kt, bt, np.ascontiguousarray(keys[rng.integers(0, 600_000, 20_000)]))
+    kt.close()

@@ -94,3 +94,16 @@ def test_full_multi_adapter_sampled():
     want = O.key_strings(kh, b"vllm@" + b"T" * 22 + b"@1@0@", 150)
     assert np.array_equal(out[torch.from_numpy(idx).cuda()].cpu().numpy(), want)
     kt.close()
+
+
+@pytest.mark.parametrize("n,width,prefix", [(200_003, 150, b"vllm@" + b"M" * 22 + b"@1@0@"), (100_001, 256, b"q" * 200),
+                                            (81_920, 22, b"")])
+def test_several_tiles_per_block(n, width, prefix):
+    """More rows than the resident CTAs hold at once (each CTA takes several
+    tiles, alternating its two shared-memory tiles): every row compared."""
+    rng = np.random.default_rng(n)
+    keys = rng.integers(0, 256, (n, 32), dtype=np.uint8)
+    got, _ = gpu_rows(keys, prefix, width)
+    want = O.key_strings(keys, prefix, width)
+    bad = np.nonzero((got != want).any(axis=1))[0]
+    assert bad.size == 0, f"{bad.size} rows differ, first {bad[:5]}"
