@@ -33,6 +33,8 @@
 //      are disjoint, so no two threads touch the same entry.
 #include <cuda_runtime.h>
 
+#include <mutex>
+
 #include "pk_device.cuh"
 #include "pk_internal.h"
 
@@ -147,9 +149,8 @@ __device__ uint64_t run_length(const uint32_t *bitmap, uint64_t s, uint64_t capa
 
 // Compaction of one cluster by one thread, serial form: in probe order an
 // evicted entry is cleared, a kept entry moves to the first empty position
-// from its home.  Any length; used for clusters longer than the planning
-// window of k_evict.
-__device__ void compact_walk(pk_entry *table, unsigned long long *stamps, uint64_t s, uint64_t L, uint64_t mask,
+// from its home.  Any length; used for clusters longer than kPlanMax.
+__device__ __noinline__ void compact_walk(pk_entry *table, unsigned long long *stamps, uint64_t s, uint64_t L, uint64_t mask,
                              unsigned long long v) {
     for (uint64_t step = 0; step < L; ++step) {
         const uint64_t pos = (s + step) & mask;
@@ -176,6 +177,105 @@ __device__ void compact_walk(pk_entry *table, unsigned long long *stamps, uint64
                 __stcg(stamps + pos, 0ull);
                 break;
             }
+        }
+    }
+}
+
+// Pending moves of one thread, flushed four at a time: the sources' entries
+// and stamps are all loaded before any target is stored.  Sources come in
+// ascending order and every target lies below its source, so no source is
+// overwritten before it is read.
+struct MoveRing {
+    uint32_t src[4], dst[4];  // positions relative to the cluster start
+    uint32_t n = 0;
+    __device__ __forceinline__ void flush(pk_entry *table, unsigned long long *stamps, uint64_t s0, uint64_t mask) {
+        uint4 kk[4], mm[4];
+        unsigned long long ss[4];
+#pragma unroll
+        for (uint32_t u = 0; u < 4; ++u) {
+            if (u < n) {
+                const uint64_t pos = (s0 + src[u]) & mask;
+                const uint4 *ep = reinterpret_cast<const uint4 *>(&table[pos]);
+                kk[u] = __ldcg(ep);
+                mm[u] = __ldcg(ep + 1);
+                ss[u] = __ldcg(stamps + pos);
+            }
+        }
+#pragma unroll
+        for (uint32_t u = 0; u < 4; ++u) {
+            if (u < n) {
+                const uint64_t t = (s0 + dst[u]) & mask;
+                uint4 *tp = reinterpret_cast<uint4 *>(&table[t]);
+                __stcg(tp + 1, mm[u]);
+                __stcg(tp, kk[u]);
+                __stcg(stamps + t, ss[u]);
+            }
+        }
+        n = 0;
+    }
+};
+
+constexpr uint32_t kPlanMax = 1024;  // longest cluster compact_planned takes
+
+// Compaction of one cluster of L <= kPlanMax entries starting at table
+// position s0 (capacity >= 64), planned as in k_evict's window: kept entries in
+// probe order take the first free position at or after their home, from the
+// evicted bits and distance bytes, 32 positions at a time.  A saturated
+// distance (255) is replaced by the exact one, from the entry's key.
+__device__ __noinline__ void compact_planned(pk_entry *table, unsigned long long *stamps, const uint32_t *evbm, const uint8_t *dist,
+                                uint64_t s0, uint32_t L, uint64_t mask) {
+    uint64_t taken[kPlanMax / 64];
+    for (uint32_t q = 0; q < kPlanMax / 64; ++q) taken[q] = 0;
+    const uint64_t n_words = (mask + 1) / 32;
+    MoveRing ring;
+    for (uint32_t c = 0; c < L; c += 32) {
+        const uint64_t p0 = (s0 + c) & mask;
+        const uint32_t off = (uint32_t)(p0 & 31);
+        const uint64_t wi = p0 >> 5;
+        uint32_t evb = __ldcg(evbm + wi) >> off;
+        if (off) evb |= __ldcg(evbm + (wi + 1) % n_words) << (32 - off);
+        uint8_t d[32];
+#pragma unroll
+        for (uint32_t k = 0; k < 32; ++k) d[k] = __ldcg(dist + ((p0 + k) & mask));
+        for (uint32_t k = 0; k < 32 && c + k < L; ++k) {
+            const uint32_t j = c + k;
+            if ((evb >> k) & 1u) continue;
+            uint64_t dd = d[k];
+            if (dd == 255) {  // saturated: the exact distance from the key (position j is not yet overwritten)
+                const uint64_t pos = (s0 + j) & mask;
+                const uint4 kj = __ldcg(reinterpret_cast<const uint4 *>(table[pos].k));
+                dd = (pos - ((((uint64_t)kj.y << 32) | kj.x) & mask)) & mask;
+            }
+            const uint32_t hh = dd <= j ? j - (uint32_t)dd : j;
+            uint32_t t = j;  // position j itself is free
+            for (uint32_t q = hh >> 6; q <= (j >> 6); ++q) {
+                uint64_t fr = ~taken[q];
+                if (q == (hh >> 6)) fr &= ~0ull << (hh & 63);
+                if (fr) {
+                    t = q * 64 + __ffsll((long long)fr) - 1;
+                    break;
+                }
+            }
+            taken[t >> 6] |= 1ull << (t & 63);
+            if (t != j) {
+                ring.src[ring.n] = j;
+                ring.dst[ring.n] = t;
+                if (++ring.n == 4) ring.flush(table, stamps, s0, mask);
+            }
+        }
+    }
+    ring.flush(table, stamps, s0, mask);
+    for (uint32_t q = 0; q * 64 < L; ++q) {  // positions left empty
+        uint64_t z = ~taken[q];
+        if (L - q * 64 < 64) z &= (1ull << (L - q * 64)) - 1ull;
+        while (z) {
+            const uint32_t p = q * 64 + __ffsll((long long)z) - 1;
+            z &= z - 1;
+            const uint64_t pos = (s0 + p) & mask;
+            uint4 *ep = reinterpret_cast<uint4 *>(&table[pos]);
+            __stcg(ep, make_uint4(0, 0, 0, 0));
+            __stcg(ep + 1, make_uint4(0, 0, 0, 0));
+            __stcg(stamps + pos, 0ull);
         }
     }
 }
@@ -388,7 +488,8 @@ k_evict(pk_entry *table, unsigned long long *stamps, uint64_t capacity, unsigned
         // 4c. compaction: one thread per bitmap word, for the clusters that start in it.  Clusters
         // that end within the 64 positions of the word and the next one are planned in registers
         // from the occupancy, evicted and distance bytes; the word's moves then go out four loads
-        // at a time.  Longer clusters (and tables below 64 entries) take compact_walk.
+        // at a time.  Longer clusters take compact_planned (the same plan, 32 positions at a time),
+        // tables below 64 entries and clusters beyond kPlanMax compact_walk.
         const unsigned long long v = prefix_v;
         const uint64_t n_words = (capacity + 31) / 32;
         for (uint64_t w = gtid; w < n_words; w += nthreads) {
@@ -439,8 +540,12 @@ k_evict(pk_entry *table, unsigned long long *stamps, uint64_t capacity, unsigned
                         }
                     }
                     zero |= (((1ull << run) - 1ull) & ~taken) << b;
-                } else {
-                    compact_walk(table, stamps, w * 32 + b, run_length(bitmap, w * 32 + b, capacity), mask, v);
+                } else {  // a longer cluster
+                    const uint64_t L = run_length(bitmap, w * 32 + b, capacity);
+                    if (L <= kPlanMax)
+                        compact_planned(table, stamps, evbm, dist, w * 32 + b, (uint32_t)L, mask);
+                    else
+                        compact_walk(table, stamps, w * 32 + b, L, mask, v);
                 }
             }
             // moves in ascending order, four loads before their stores: a target is below its
@@ -495,17 +600,33 @@ uint64_t pk_evict_scratch_bytes_impl(uint64_t capacity) {
     return kHeaderBytes + 2 * bitmap_bytes(capacity) + 8 * capacity + 4 * capacity + ((capacity + 255) & ~255ull);
 }
 
+// Resident CTAs of k_evict on a device (SMs x CTAs per SM), computed once per device.
+static cudaError_t evict_resident(int dev, uint64_t *out) {
+    static std::mutex mu;
+    static uint64_t cache[256] = {};
+    if (dev < 0 || dev >= 256) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!cache[dev]) {
+        int sms = 0, per_sm = 0;
+        cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_evict, kEvThreads, 0);
+        if (e != cudaSuccess) return e;
+        if (per_sm < 1) return cudaErrorInvalidConfiguration;
+        cache[dev] = (uint64_t)sms * per_sm;
+    }
+    *out = cache[dev];
+    return cudaSuccess;
+}
+
 cudaError_t pk_launch_evict(const pk_ctx *ctx, uint64_t budget, uint64_t keep, void *scratch, uint32_t *evicted,
                             uint64_t evicted_cap, unsigned long long *n_evicted, int32_t *status, cudaStream_t s) {
-    int dev = 0, sms = 0, per_sm = 0;
+    int dev = 0;
+    uint64_t resident = 0;
     cudaError_t e = cudaGetDevice(&dev);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_evict, kEvThreads, 0);
+    if (e == cudaSuccess) e = evict_resident(dev, &resident);
     if (e != cudaSuccess) return e;
-    if (per_sm < 1) return cudaErrorInvalidConfiguration;
     // every CTA resident (the barriers need it); no more CTAs than the table has rows of kEvThreads entries
     const uint64_t want = (ctx->capacity + kEvThreads - 1) / kEvThreads;
-    const uint64_t resident = (uint64_t)sms * per_sm;
     const unsigned grid = (unsigned)(want < resident ? want : resident);
     uint8_t *base = static_cast<uint8_t *>(scratch);
     EvictHeader *h = reinterpret_cast<EvictHeader *>(base);

@@ -20,6 +20,8 @@
 // ahead.
 #include <cuda_runtime.h>
 
+#include <mutex>
+
 #include "pk_device.cuh"
 #include "pk_internal.h"
 
@@ -111,6 +113,34 @@ __global__ void __launch_bounds__(kRows) k_key_strings(const uint8_t *keys, uint
 
 }  // namespace
 
+// Resident CTAs of k_key_strings for a row width (SMs x CTAs per SM), computed
+// once per device and width; the first call also raises the kernel's dynamic
+// shared-memory limit to the largest width's two tiles.
+static cudaError_t keystr_resident(int dev, uint32_t width, uint64_t *out) {
+    static std::mutex mu;
+    static uint32_t sms[256] = {};
+    static uint16_t per_sm[256][PK_KEY_STRING_MAX_WIDTH + 1] = {};
+    if (dev < 0 || dev >= 256 || width > PK_KEY_STRING_MAX_WIDTH) return cudaErrorInvalidValue;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!sms[dev]) {
+        int n = 0;
+        cudaError_t e = cudaFuncSetAttribute(k_key_strings, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)(2 * kRows * PK_KEY_STRING_MAX_WIDTH));
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return e;
+        sms[dev] = (uint32_t)n;
+    }
+    if (!per_sm[dev][width]) {
+        int b = 0;
+        const cudaError_t e =
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, k_key_strings, kRows, 2ull * kRows * width);
+        if (e != cudaSuccess) return e;
+        per_sm[dev][width] = (uint16_t)(b < 1 ? 1 : b);
+    }
+    *out = (uint64_t)sms[dev] * per_sm[dev][width];
+    return cudaSuccess;
+}
+
 cudaError_t pk_launch_key_strings(const uint8_t *keys, uint64_t n, const uint8_t *prefix, uint32_t plen,
                                   uint32_t width, uint8_t *out, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
@@ -119,16 +149,12 @@ cudaError_t pk_launch_key_strings(const uint8_t *keys, uint64_t n, const uint8_t
     a.width = width;
     for (uint32_t j = 0; j < PK_KEY_STRING_MAX_WIDTH; ++j) a.prefix[j] = j < plen ? prefix[j] : 0;
     const size_t smem = 2ull * kRows * width;  // <= 128 KiB
-    cudaError_t e = cudaFuncSetAttribute(k_key_strings, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)(2 * kRows * PK_KEY_STRING_MAX_WIDTH));
-    int dev = 0, sms = 0, per_sm = 0;
-    if (e == cudaSuccess) e = cudaGetDevice(&dev);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_key_strings, kRows, smem);
+    int dev = 0;
+    uint64_t resident = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = keystr_resident(dev, width, &resident);
     if (e != cudaSuccess) return e;
-    if (per_sm < 1) per_sm = 1;
     const uint64_t tiles = (n + kRows - 1) / kRows;
-    const uint64_t resident = (uint64_t)sms * per_sm;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(tiles < resident ? tiles : resident));
     cfg.blockDim = dim3(kRows);
