@@ -511,12 +511,18 @@ int pk_table_load(pk_ctx *ctx, const void *src, size_t src_bytes, pk_stream stre
     const size_t tb = pk_table_bytes(ctx->capacity_log2);
     if (src_bytes < tb + 64) return PK_ERR_ARG;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (ctx->epoch < 1) ctx->epoch = 1;
+    if (ctx->stamps && cudaMemsetAsync(ctx->stamps, 0, 8ull * ctx->capacity, s) != cudaSuccess) return PK_ERR_CUDA;
+    cudaPointerAttributes attr;
+    const bool on_device = cudaPointerGetAttributes(&attr, src) == cudaSuccess &&
+                           (attr.type == cudaMemoryTypeDevice || attr.type == cudaMemoryTypeManaged) &&
+                           aligned16(src);
+    if (!on_device) cudaGetLastError();  // (a host pointer may leave an error from the query)
+    if (on_device) return cuda_rc(pk_launch_load_table(ctx, src, s));  // one pass, copy and mark
     if (cudaMemcpyAsync(ctx->table, src, tb, cudaMemcpyDefault, s) != cudaSuccess ||
         cudaMemcpyAsync(ctx->counter_dev, static_cast<const uint8_t *>(src) + tb, sizeof(unsigned long long),
                         cudaMemcpyDefault, s) != cudaSuccess)
         return PK_ERR_CUDA;
-    if (ctx->epoch < 1) ctx->epoch = 1;
-    if (ctx->stamps && cudaMemsetAsync(ctx->stamps, 0, 8ull * ctx->capacity, s) != cudaSuccess) return PK_ERR_CUDA;
     return cuda_rc(pk_launch_mark_loaded(ctx, s));
 }
 

@@ -56,6 +56,7 @@ cudaError_t pk_launch_store_noalloc(pk_entry *table, uint32_t capacity_log2, uin
                                     const int32_t *hit_chunks, uint32_t R, int32_t *result, uint32_t *slot_out,
                                     int32_t *status, cudaStream_t s);
 cudaError_t pk_launch_mark_loaded(const pk_ctx *ctx, cudaStream_t s);
+cudaError_t pk_launch_load_table(const pk_ctx *ctx, const void *src, cudaStream_t s);
 cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const uint8_t *keys,
                             const uint32_t *slots, uint64_t n, const int64_t *key_off,
                             const int32_t *hit_chunks, uint32_t R, int32_t *result, uint32_t *slot_out,

@@ -954,8 +954,35 @@ k_store_finalize(const pk_entry *table, uint64_t n, const int64_t *key_off, uint
     slot_out[e] = (uint32_t)w;
 }
 
-// After a table load: every stored entry counts as inserted before any later
-// store call (epoch 1; calls on this context use epochs >= 2 from then on).
+// Table load from device memory in one pass: each 32-byte entry copied whole
+// (full-sector writes), a stored entry marked as inserted before any later
+// store call (epoch 1, owner 0), and the entry count copied by thread 0.  One
+// entry per thread: short blocks, so that kernels of other streams find free
+// SM slots while a table is restored beside them.
+__global__ void __launch_bounds__(256) k_load_table(pk_entry *table, const pk_entry *src, uint64_t capacity,
+                                                    unsigned long long *counter, const unsigned long long *src_count) {
+    pk::pdl_wait(table, src, counter, src_count);
+    const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i == 0) *counter = __ldcg(src_count);
+    if (i < capacity) {
+        const uint4 *sp = reinterpret_cast<const uint4 *>(&src[i]);
+        const uint4 k = __ldcg(sp);
+        uint4 m = __ldcg(sp + 1);  // slot, owner, epoch (low, high)
+        if (!is_zero(k)) {
+            m.y = 0u;
+            m.z = 1u;
+            m.w = 0u;
+        }
+        uint4 *tp = reinterpret_cast<uint4 *>(&table[i]);
+        tp[0] = k;
+        tp[1] = m;
+    }
+    pk::pdl_launch_dependents();
+}
+
+// After a table load from host memory: every stored entry counts as inserted
+// before any later store call (epoch 1; calls on this context use epochs >= 2
+// from then on).
 __global__ void k_mark_loaded(pk_entry *table, uint64_t capacity) {
     for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < capacity;
          i += (uint64_t)gridDim.x * blockDim.x) {
@@ -1065,6 +1092,16 @@ unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1
 bool per_request(uint32_t R, uint64_t key_capacity) { return R >= 1024 || key_capacity <= 64ull * R; }
 
 }  // namespace
+
+cudaError_t pk_launch_load_table(const pk_ctx *ctx, const void *src, cudaStream_t s) {
+    const uint64_t blocks = (ctx->capacity + 255) / 256;  // <= 2^23
+    const pk_entry *sp = static_cast<const pk_entry *>(src);
+    const unsigned long long *cp =
+        reinterpret_cast<const unsigned long long *>(static_cast<const uint8_t *>(src) + PK_ENTRY_BYTES * ctx->capacity);
+    const cudaError_t e = pk_launch(k_load_table, (unsigned)blocks, 256, s, ctx->table, sp, ctx->capacity,
+                                    ctx->counter_dev, cp);
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
 
 cudaError_t pk_launch_mark_loaded(const pk_ctx *ctx, cudaStream_t s) {
     const uint64_t blocks = (ctx->capacity + 255) / 256;
