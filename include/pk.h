@@ -253,6 +253,19 @@ int pk_lookup_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_
                     uint32_t R, uint64_t key_capacity, int32_t *hit_chunks_dev, uint32_t *slots_dev,
                     int32_t *result_dev, uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream);
 
+/* Device.  The whole hot path in one call (a0-a4): pk_derive_keys_enc
+ * followed by pk_lookup_store on its keys, enqueued together.  Arguments as
+ * the two calls (tokens ... key_capacity as pk_derive_keys_enc; slots_new_dev,
+ * hit_chunks_dev, slots_dev, result_dev, slot_out_dev as pk_lookup_store);
+ * outputs, results and device errors equal those of the two calls (one store
+ * call number); all host checks run before anything is enqueued. */
+int pk_derive_lookup_store(pk_ctx *ctx, const int32_t *tokens_dev, uint64_t n_tokens, const int64_t *tok_off_dev,
+                           uint32_t R, const uint32_t *desc_idx_dev, const uint8_t *enc_dev, uint64_t enc_bytes,
+                           const int64_t *enc_off_dev, uint32_t D, uint8_t *digests_dev, int64_t *key_off_dev,
+                           uint8_t *keys_dev, uint64_t key_capacity, const uint32_t *slots_new_dev,
+                           int32_t *hit_chunks_dev, uint32_t *slots_dev, int32_t *result_dev, uint32_t *slot_out_dev,
+                           int32_t *status_dev, pk_stream stream);
+
 /* Device.  The comparison step of the store-side differential omission test
  * (Sec. 6.3, omission detection; Eq. 4): a worker's keys joined to a
  * reference worker's by pk_lookup on a table holding the reference keys

@@ -420,6 +420,38 @@ int pk_key_strings(const uint8_t *keys_dev, uint64_t n, const char *prefix, uint
                                          reinterpret_cast<uint8_t *>(out_dev), reinterpret_cast<cudaStream_t>(stream)));
 }
 
+int pk_derive_lookup_store(pk_ctx *ctx, const int32_t *tokens_dev, uint64_t n_tokens, const int64_t *tok_off_dev,
+                           uint32_t R, const uint32_t *desc_idx_dev, const uint8_t *enc_dev, uint64_t enc_bytes,
+                           const int64_t *enc_off_dev, uint32_t D, uint8_t *digests_dev, int64_t *key_off_dev,
+                           uint8_t *keys_dev, uint64_t key_capacity, const uint32_t *slots_new_dev,
+                           int32_t *hit_chunks_dev, uint32_t *slots_dev, int32_t *result_dev, uint32_t *slot_out_dev,
+                           int32_t *status_dev, pk_stream stream) {
+    // the checks of pk_derive_keys_enc ...
+    if (!ctx || !tok_off_dev || !key_off_dev) return PK_ERR_ARG;
+    if (n_tokens && !tokens_dev) return PK_ERR_ARG;
+    if (R && (!desc_idx_dev || D == 0 || !hit_chunks_dev)) return PK_ERR_ARG;
+    if (D && (!enc_off_dev || !digests_dev || !aligned16(digests_dev) || !aligned(enc_off_dev, 8))) return PK_ERR_ARG;
+    if (enc_bytes && !enc_dev) return PK_ERR_ARG;
+    if (key_capacity < n_tokens / ctx->chunk_tokens) return PK_ERR_ARG;
+    if (key_capacity && (!keys_dev || !aligned16(keys_dev))) return PK_ERR_ARG;
+    if (!aligned(tokens_dev, 4) || !aligned(tok_off_dev, 8) || !aligned(desc_idx_dev, 4) || !aligned(key_off_dev, 8))
+        return PK_ERR_ARG;
+    // ... and of pk_lookup_store
+    if (key_capacity && (!slots_new_dev || !slots_dev || !result_dev || !slot_out_dev)) return PK_ERR_ARG;
+    if (key_capacity > (uint64_t)0x7fffffff * 64 || key_capacity >= 0xffffffffull) return PK_ERR_ARG;
+    if (!aligned(hit_chunks_dev, 4) || !aligned(slots_new_dev, 4) || !aligned(slots_dev, 4) || !aligned(result_dev, 4) ||
+        !aligned(slot_out_dev, 4))
+        return PK_ERR_ARG;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = pk_launch_derive_enc(ctx, tokens_dev, n_tokens, tok_off_dev, R, desc_idx_dev, enc_dev, enc_bytes,
+                                         D ? enc_off_dev : nullptr, D, digests_dev, key_off_dev, keys_dev, key_capacity,
+                                         status_dev, s);
+    if (e != cudaSuccess) return PK_ERR_CUDA;
+    const unsigned long long epoch = ++ctx->epoch;
+    return cuda_rc(pk_launch_lookup_store(ctx, epoch, keys_dev, slots_new_dev, key_off_dev, R, key_capacity,
+                                          hit_chunks_dev, slots_dev, result_dev, slot_out_dev, status_dev, s));
+}
+
 int pk_compare_pages(const uint32_t *slots_dev, const uint8_t *pages_dev, const uint8_t *ref_pages_dev, uint64_t n,
                      uint64_t n_ref, uint64_t page_bytes, int32_t *verdict_dev, uint64_t *counts_dev,
                      int32_t *status_dev, pk_stream stream) {

@@ -94,6 +94,8 @@ def lib() -> ctypes.CDLL:
             "pk_lookup": (ctypes.c_int, [_VP, _VP, _VP, _U32, _U64, _VP, _VP, _VP, _VP]),
             "pk_store": (ctypes.c_int, [_VP, _VP, _VP, _U64, _VP, _VP, _U32, _VP, _VP, _VP, _VP]),
             "pk_lookup_store": (ctypes.c_int, [_VP, _VP, _VP, _VP, _U32, _U64, _VP, _VP, _VP, _VP, _VP, _VP]),
+            "pk_derive_lookup_store": (ctypes.c_int, [_VP, _VP, _U64, _VP, _U32, _VP, _VP, _U64, _VP, _U32, _VP, _VP,
+                                                      _VP, _U64, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
             "pk_entries": (ctypes.c_int, [_VP, ctypes.POINTER(ctypes.c_uint64), _VP]),
             "pk_store_noalloc": (ctypes.c_int, [ctypes.POINTER(pk_config), _VP, _VP, _U64, _VP, _VP, _U32, _VP, _VP,
                                                 _VP, _VP]),
@@ -324,6 +326,18 @@ def pk_lookup_store(ctx: int, keys: torch.Tensor, new_slots: torch.Tensor, key_o
     _check(lib().pk_lookup_store(ctx, _p(keys), _p(new_slots), _p(key_off), R, keys.numel() // 32,
                                  _p(hit_chunks), _p(slots), _p(result), _p(slot_out), _p(status), _s(stream)),
            "pk_lookup_store")
+
+
+def pk_derive_lookup_store(ctx: int, tokens: torch.Tensor, tok_off: torch.Tensor, desc_idx: torch.Tensor,
+                           enc: torch.Tensor, enc_off: torch.Tensor, digests: torch.Tensor, key_off: torch.Tensor,
+                           keys: torch.Tensor, new_slots: torch.Tensor, hit_chunks: torch.Tensor, slots: torch.Tensor,
+                           result: torch.Tensor, slot_out: torch.Tensor, status: torch.Tensor, stream=None) -> None:
+    R = tok_off.numel() - 1
+    D = enc_off.numel() - 1
+    _check(lib().pk_derive_lookup_store(ctx, _p(tokens), tokens.numel(), _p(tok_off), R, _p(desc_idx), _p(enc),
+                                        enc.numel(), _p(enc_off), D, _p(digests), _p(key_off), _p(keys),
+                                        keys.numel() // 32, _p(new_slots), _p(hit_chunks), _p(slots), _p(result),
+                                        _p(slot_out), _p(status), _s(stream)), "pk_derive_lookup_store")
 
 
 def pk_compare_pages(slots: torch.Tensor, pages: torch.Tensor, ref_pages: torch.Tensor, verdict: torch.Tensor,

@@ -159,6 +159,31 @@ class KeyTable:
                            self.stream)
         return hit, slots, result, slot_out
 
+    def derive_lookup_store(self, tokens, tok_off, desc_idx, descriptors, new_slots):
+        """The whole hot path in one call (pk_derive_lookup_store): returns
+        (digests, key_off, keys, hit, slots, result, slot_out)."""
+        enc, off = pk.pk_descriptors_encode(descriptors)
+        D = off.size - 1
+        enc_d = _dev(enc if enc.size else np.zeros(1, np.uint8), torch.uint8, self.device)[: enc.size]
+        off_d = _dev(off, torch.int64, self.device)
+        digests = torch.zeros((max(D, 1), 32), dtype=torch.uint8, device=self.device)[:D]
+        tokens = _dev(tokens, torch.int32, self.device)
+        tok_off = _dev(tok_off, torch.int64, self.device)
+        desc_idx = _dev(desc_idx, torch.int32, self.device)
+        R = tok_off.numel() - 1
+        cap = tokens.numel() // self.chunk_tokens
+        key_off = torch.empty(R + 1, dtype=torch.int64, device=self.device)
+        keys = torch.empty((max(cap, 0), 32), dtype=torch.uint8, device=self.device)
+        new_slots = _dev(new_slots if isinstance(new_slots, torch.Tensor) else np.asarray(new_slots, np.uint32),
+                         torch.int32, self.device)
+        hit = torch.empty(R, dtype=torch.int32, device=self.device)
+        slots = torch.empty(max(cap, 0), dtype=torch.int32, device=self.device)
+        result = torch.empty(max(cap, 0), dtype=torch.int32, device=self.device)
+        slot_out = torch.empty(max(cap, 0), dtype=torch.int32, device=self.device)
+        pk.pk_derive_lookup_store(self.ctx, tokens, tok_off, desc_idx, enc_d, off_d, digests, key_off, keys, new_slots,
+                                  hit, slots, result, slot_out, self.status, self.stream)
+        return digests, key_off, keys, hit, slots, result, slot_out
+
     # -- budget mode (eviction under a fixed budget) -------------------------
     def attach_stamps(self) -> torch.Tensor:
         """Turn budget mode on: a zeroed last-use stamp per entry, and the
