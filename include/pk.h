@@ -305,6 +305,16 @@ int pk_compare_pages(const uint32_t *slots_dev, const uint8_t *pages_dev, const 
 size_t pk_content_scratch_bytes(uint64_t n_bytes);
 int pk_content_digest(const uint8_t *bytes_dev, uint64_t n_bytes, uint8_t *scratch_dev, size_t scratch_bytes,
                       uint8_t *top_dev, pk_stream stream);
+/* The same for n buffers at once (an adapter's tensors): tops_dev[32 j ..]
+ * = the tree top of bytes_dev[j][0, n_bytes[j]).  bytes_dev and n_bytes are
+ * host arrays of n entries (device pointers, 16-byte aligned); every tree
+ * level of all the buffers (128 at a time) is one launch, so a call costs
+ * about as many launches as its largest buffer has levels.  scratch_dev:
+ * pk_content_scratch_bytes_batch(n_bytes, n) bytes, 16-byte aligned.
+ * Errors: PK_ERR_ARG (host), PK_ERR_CUDA. */
+size_t pk_content_scratch_bytes_batch(const uint64_t *n_bytes, uint32_t n);
+int pk_content_digests(const uint8_t *const *bytes_dev, const uint64_t *n_bytes, uint32_t n, uint8_t *scratch_dev,
+                       size_t scratch_bytes, uint8_t *tops_dev, pk_stream stream);
 int pk_tensor_identity(const pk_bytes *name, const pk_bytes *dtype, const int64_t *shape, uint32_t ndim,
                        uint64_t n_bytes, const uint8_t top[32], uint8_t out[32]);
 int pk_adapter_identity(const uint8_t *tensor_ids, uint32_t n_tensors, const pk_bytes *config, uint32_t n_config,

@@ -19,6 +19,15 @@ namespace {
 constexpr int kTreeThreads = 128;
 constexpr uint64_t kTreeBlock = 1024;  // bytes per tree block
 
+// 16-byte L2 load kept in program order (a prefetch the compiler must not sink).
+__device__ __forceinline__ uint4 ld_cg_v4_ordered(const void *p) {
+    uint4 v;
+    asm volatile("ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
 // 16 big-endian message words of bytes [off, off + 64) of src, zero past n.
 __device__ __forceinline__ void load_words(const uint8_t *src, uint64_t n, uint64_t off, uint32_t w[16]) {
 #pragma unroll
@@ -26,7 +35,7 @@ __device__ __forceinline__ void load_words(const uint8_t *src, uint64_t n, uint6
         const uint64_t o = off + 16 * v;
         uint4 x = make_uint4(0, 0, 0, 0);
         if (o + 16 <= n) {
-            x = __ldcg(reinterpret_cast<const uint4 *>(src + o));
+            x = ld_cg_v4_ordered(src + o);
         } else if (o < n) {  // the buffer's last partial 16 bytes
             uint32_t b[4] = {0, 0, 0, 0};
             for (uint64_t k = o; k < n; ++k) b[(k - o) / 4] |= (uint32_t)src[k] << (8 * ((k - o) % 4));
@@ -39,21 +48,46 @@ __device__ __forceinline__ void load_words(const uint8_t *src, uint64_t n, uint6
     }
 }
 
-// dst[t] = SHA-256 of block t (1 KiB) of src[0, n), zero-padded, t < m.
-__global__ void __launch_bounds__(kTreeThreads)
-k_tree_level(const uint8_t *src, uint64_t n, uint8_t *dst, uint64_t m) {
+// One tree level of up to kMaxSeg buffers in one launch: segment j hashes the
+// 1 KiB blocks of src[0, n) (zero-padded) into dst, its blocks being the
+// launch's threads first[j] .. first[j+1]-1 (the segments passed by value stay
+// within the 4 KiB kernel-parameter space).
+constexpr uint32_t kMaxSeg = 128;
+struct TreeSeg {
+    const uint8_t *src;
+    uint64_t n;
+    uint8_t *dst;
+};
+struct TreeLevel {
+    uint32_t count;
+    uint32_t first[kMaxSeg + 1];  // first[count] = threads of the launch
+    TreeSeg seg[kMaxSeg];
+};
+static_assert(sizeof(TreeLevel) <= 4000, "kernel parameter space");
+
+__global__ void __launch_bounds__(kTreeThreads) k_tree_level(const TreeLevel lv) {
     __shared__ uint32_t sK[64];
     if (threadIdx.x < 64) sK[threadIdx.x] = pk::kSha256K[threadIdx.x];
     __syncthreads();
-    pk::pdl_wait(src, dst);
+    pk::pdl_wait();
     const uint64_t t = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (t < m) {
-        uint32_t st[8], w[16];
+    if (t < lv.first[lv.count]) {
+        uint32_t lo = 0, hi = lv.count;  // first[lo] <= t < first[hi]
+        while (hi - lo > 1) {
+            const uint32_t mid = (lo + hi) >> 1;
+            if (lv.first[mid] <= t) lo = mid; else hi = mid;
+        }
+        const TreeSeg sg = lv.seg[lo];
+        const uint64_t b = t - lv.first[lo];
+        uint32_t st[8], w[16], wn[16];
         pk::init_state(st);
-        const uint64_t base = t * kTreeBlock;
+        const uint64_t base = b * kTreeBlock;
+        load_words(sg.src, sg.n, base, wn);
 #pragma unroll 1
-        for (uint64_t b = 0; b < kTreeBlock / 64; ++b) {
-            load_words(src, n, base + 64 * b, w);
+        for (uint64_t q = 0; q < kTreeBlock / 64; ++q) {  // the next 64 bytes load while these are compressed
+#pragma unroll
+            for (int k = 0; k < 16; ++k) w[k] = wn[k];
+            if (q + 1 < kTreeBlock / 64) load_words(sg.src, sg.n, base + 64 * (q + 1), wn);
             pk::compress_rolled(st, w, sK);
         }
         // padding of a 1024-byte message: 0x80, zeros, the length in bits (8192)
@@ -62,7 +96,7 @@ k_tree_level(const uint8_t *src, uint64_t n, uint8_t *dst, uint64_t m) {
         w[0] = 0x80000000u;
         w[15] = (uint32_t)(kTreeBlock * 8);
         pk::compress_rolled(st, w, sK);
-        uint4 *q = reinterpret_cast<uint4 *>(dst + 32 * t);
+        uint4 *q = reinterpret_cast<uint4 *>(sg.dst + 32 * b);
         q[0] = make_uint4(pk::bswap32(st[0]), pk::bswap32(st[1]), pk::bswap32(st[2]), pk::bswap32(st[3]));
         q[1] = make_uint4(pk::bswap32(st[4]), pk::bswap32(st[5]), pk::bswap32(st[6]), pk::bswap32(st[7]));
     }
@@ -83,21 +117,57 @@ uint64_t pk_content_scratch_bytes_impl(uint64_t n_bytes) {
     return total;
 }
 
-cudaError_t pk_launch_content_digest(const uint8_t *bytes, uint64_t n_bytes, uint8_t *scratch, uint8_t *top,
-                                     cudaStream_t s) {
-    const uint8_t *src = bytes;
-    uint64_t n = n_bytes, m = blocks_of(n_bytes);
-    uint8_t *dst = scratch;
-    while (true) {
-        uint8_t *out = m == 1 ? top : dst;
-        const cudaError_t e = pk_launch(k_tree_level, (unsigned)((m + kTreeThreads - 1) / kTreeThreads),
-                                        kTreeThreads, s, src, n, out, m);
-        if (e != cudaSuccess) return e;
-        if (m == 1) break;
-        src = dst;
-        n = 32 * m;
-        dst += 32 * m;
-        m = blocks_of(n);
+// Tree tops of n buffers: every level of every buffer not yet reduced to one
+// digest in one launch per level (kMaxSeg buffers at a time).  Buffer j's
+// levels go to scratch at scratch_off[j]; its last level writes tops[32 j].
+cudaError_t pk_launch_content_digests(const uint8_t *const *bytes, const uint64_t *n_bytes, uint32_t n,
+                                      uint8_t *scratch, const uint64_t *scratch_off, uint8_t *tops, cudaStream_t s) {
+    for (uint32_t j0 = 0; j0 < n; j0 += kMaxSeg) {
+        const uint32_t cnt = n - j0 < kMaxSeg ? n - j0 : kMaxSeg;
+        TreeSeg cur[kMaxSeg];
+        uint64_t m[kMaxSeg];
+        bool done[kMaxSeg];
+        for (uint32_t j = 0; j < cnt; ++j) {
+            cur[j] = TreeSeg{bytes[j0 + j], n_bytes[j0 + j], scratch + scratch_off[j0 + j]};
+            m[j] = blocks_of(n_bytes[j0 + j]);
+            done[j] = false;
+        }
+        for (;;) {
+            TreeLevel lv;
+            lv.count = 0;
+            uint64_t threads = 0;
+            for (uint32_t j = 0; j < cnt; ++j) {
+                if (done[j]) continue;
+                TreeSeg sg = cur[j];
+                if (m[j] == 1) sg.dst = tops + 32ull * (j0 + j);
+                lv.first[lv.count] = (uint32_t)threads;
+                lv.seg[lv.count++] = sg;
+                threads += m[j];
+            }
+            if (lv.count == 0) break;
+            if (threads >= (1ull << 31)) return cudaErrorInvalidValue;
+            lv.first[lv.count] = (uint32_t)threads;
+            const cudaError_t e =
+                pk_launch(k_tree_level, (unsigned)((threads + kTreeThreads - 1) / kTreeThreads), kTreeThreads, s, lv);
+            if (e != cudaSuccess) return e;
+            for (uint32_t j = 0; j < cnt; ++j) {  // the next level reads this one
+                if (done[j]) continue;
+                if (m[j] == 1) {
+                    done[j] = true;
+                    continue;
+                }
+                cur[j].src = cur[j].dst;
+                cur[j].n = 32 * m[j];
+                cur[j].dst += 32 * m[j];
+                m[j] = blocks_of(cur[j].n);
+            }
+        }
     }
     return cudaGetLastError();
+}
+
+cudaError_t pk_launch_content_digest(const uint8_t *bytes, uint64_t n_bytes, uint8_t *scratch, uint8_t *top,
+                                     cudaStream_t s) {
+    const uint64_t off = 0;
+    return pk_launch_content_digests(&bytes, &n_bytes, 1, scratch, &off, top, s);
 }

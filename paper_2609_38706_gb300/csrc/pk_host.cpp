@@ -7,6 +7,7 @@
 #include <cstring>
 #include <new>
 #include <string>
+#include <vector>
 
 #include "pk_internal.h"
 #include "pk_sha256.cuh"
@@ -474,6 +475,30 @@ int pk_content_digest(const uint8_t *bytes_dev, uint64_t n_bytes, uint8_t *scrat
     if (scratch_bytes < pk_content_scratch_bytes_impl(n_bytes)) return PK_ERR_ARG;
     return cuda_rc(pk_launch_content_digest(bytes_dev, n_bytes, scratch_dev, top_dev,
                                             reinterpret_cast<cudaStream_t>(stream)));
+}
+
+size_t pk_content_scratch_bytes_batch(const uint64_t *n_bytes, uint32_t n) {
+    if (n && !n_bytes) return 0;
+    uint64_t total = 0;
+    for (uint32_t j = 0; j < n; ++j) total += (pk_content_scratch_bytes_impl(n_bytes[j]) + 15) & ~15ull;
+    return (size_t)total;
+}
+
+int pk_content_digests(const uint8_t *const *bytes_dev, const uint64_t *n_bytes, uint32_t n, uint8_t *scratch_dev,
+                       size_t scratch_bytes, uint8_t *tops_dev, pk_stream stream) {
+    if (n == 0) return PK_OK;
+    if (!bytes_dev || !n_bytes || !scratch_dev || !tops_dev || !aligned16(scratch_dev) || !aligned16(tops_dev))
+        return PK_ERR_ARG;
+    std::vector<uint64_t> off(n);
+    uint64_t total = 0;
+    for (uint32_t j = 0; j < n; ++j) {
+        if ((n_bytes[j] && !bytes_dev[j]) || !aligned16(bytes_dev[j])) return PK_ERR_ARG;
+        off[j] = total;
+        total += (pk_content_scratch_bytes_impl(n_bytes[j]) + 15) & ~15ull;
+    }
+    if (scratch_bytes < total) return PK_ERR_ARG;
+    return cuda_rc(pk_launch_content_digests(bytes_dev, n_bytes, n, scratch_dev, off.data(), tops_dev,
+                                             reinterpret_cast<cudaStream_t>(stream)));
 }
 
 int pk_tensor_identity(const pk_bytes *name, const pk_bytes *dtype, const int64_t *shape, uint32_t ndim,

@@ -64,6 +64,8 @@ cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const u
 uint64_t pk_content_scratch_bytes_impl(uint64_t n_bytes);
 cudaError_t pk_launch_content_digest(const uint8_t *bytes, uint64_t n_bytes, uint8_t *scratch, uint8_t *top,
                                      cudaStream_t s);
+cudaError_t pk_launch_content_digests(const uint8_t *const *bytes, const uint64_t *n_bytes, uint32_t n,
+                                      uint8_t *scratch, const uint64_t *scratch_off, uint8_t *tops, cudaStream_t s);
 cudaError_t pk_launch_compare_pages(const uint32_t *slots, const uint8_t *pages, const uint8_t *ref_pages, uint64_t n,
                                     uint64_t n_ref, uint64_t page_bytes, int32_t *verdict, unsigned long long *counts,
                                     int32_t *status, cudaStream_t s);

@@ -102,6 +102,8 @@ def lib() -> ctypes.CDLL:
             "pk_compare_pages": (ctypes.c_int, [_VP, _VP, _VP, _U64, _U64, _U64, _VP, _VP, _VP, _VP]),
             "pk_content_scratch_bytes": (ctypes.c_size_t, [_U64]),
             "pk_content_digest": (ctypes.c_int, [_VP, _U64, _VP, ctypes.c_size_t, _VP, _VP]),
+            "pk_content_scratch_bytes_batch": (ctypes.c_size_t, [_VP, _U32]),
+            "pk_content_digests": (ctypes.c_int, [_VP, _VP, _U32, _VP, ctypes.c_size_t, _VP, _VP]),
             "pk_tensor_identity": (ctypes.c_int, [ctypes.POINTER(pk_bytes), ctypes.POINTER(pk_bytes), _VP, _U32,
                                                   _U64, _VP, _VP]),
             "pk_adapter_identity": (ctypes.c_int, [_VP, _U32, ctypes.POINTER(pk_bytes), _U32, _VP]),
@@ -357,6 +359,20 @@ def pk_content_digest(data: torch.Tensor, scratch: torch.Tensor, top: torch.Tens
     n = data.numel() * data.element_size()
     _check(lib().pk_content_digest(_p(data), n, _p(scratch), scratch.numel(), _p(top), _s(stream)),
            "pk_content_digest")
+
+
+def pk_content_scratch_bytes_batch(sizes) -> int:
+    arr = (ctypes.c_uint64 * max(len(sizes), 1))(*[int(x) for x in sizes])
+    return int(lib().pk_content_scratch_bytes_batch(arr, len(sizes)))
+
+
+def pk_content_digests(datas, scratch: torch.Tensor, tops: torch.Tensor, stream=None) -> None:
+    """tops (uint8[n, 32], device) = the tree tops of the contiguous device tensors `datas`."""
+    n = len(datas)
+    ptrs = (ctypes.c_void_p * max(n, 1))(*[_p(d) for d in datas])
+    sizes = (ctypes.c_uint64 * max(n, 1))(*[d.numel() * d.element_size() for d in datas])
+    _check(lib().pk_content_digests(ptrs, sizes, n, _p(scratch), scratch.numel(), _p(tops), _s(stream)),
+           "pk_content_digests")
 
 
 def _pkb(b: bytes):
