@@ -160,7 +160,26 @@ def oracle_setup(wl):
     return d_ref, table
 
 
+def _hashlib_keys(task):
+    """Worker of the hashlib baseline (a spawned process): the keys of requests [r0, r1)."""
+    import oracle as O
+    tokens, tok_off, C, desc_idx, digests, r0, r1 = task
+    return O.derive_keys_hashlib(tokens, tok_off, C, desc_idx, digests, range(r0, r1)).shape[0]
+
+
+def keys_rate(fn, wl, seconds: float):
+    """Full-chunk tokens per second of fn() (one batch's keys per call), over about `seconds`."""
+    n, t0 = 0, time.perf_counter()
+    while True:
+        fn()
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            return wl.tokens_keyed() * n / el, n, el
+
+
 def run_cpu_baseline(wl, seconds: float) -> dict:
+    import multiprocessing
     import oracle as O
     d_ref, table = oracle_setup(wl)
     n0 = len(table)
@@ -171,10 +190,50 @@ def run_cpu_baseline(wl, seconds: float) -> dict:
         el = time.perf_counter() - t0
         if el >= seconds or passes >= 1000:
             break
-    return {"value": wl.tokens_keyed() * passes / el, "unit": "tokens/s", "cores": O.max_threads(),
+    cores = O.max_threads()
+    b = wl.batch
+    part = max(seconds / 3, 1.0)
+    # key derivation alone: the C oracle on one thread and on every core, and the standard library's
+    # SHA-256 (OpenSSL) over a spawned process per core
+    derive = lambda: O.derive_keys(b.tokens, b.tok_off, wl.chunk_tokens, b.desc_idx, d_ref)
+    O.set_threads(1)
+    one, n1, e1 = keys_rate(derive, wl, part)
+    O.set_threads(cores)
+    omp, n2, e2 = keys_rate(derive, wl, part)
+    bounds = np.linspace(0, b.R, 4 * cores + 1).astype(int)
+    tasks = [(b.tokens[b.tok_off[r0]:b.tok_off[r1]], b.tok_off[r0:r1 + 1] - b.tok_off[r0], wl.chunk_tokens,
+              b.desc_idx[r0:r1], d_ref, 0, r1 - r0) for r0, r1 in zip(bounds[:-1], bounds[1:])]
+    hl, n3, e3, why = None, 0, 0.0, ""
+    try:  # every wait on the pool is bounded: a pool that cannot start reports null
+        with multiprocessing.get_context("spawn").Pool(cores) as pool:
+            pool.map_async(_hashlib_keys, tasks[:cores]).get(timeout=120)  # start-up outside the timing
+            hl, n3, e3 = keys_rate(lambda: pool.map_async(_hashlib_keys, tasks).get(timeout=120), wl, part)
+    except Exception as exc:  # (multiprocessing.TimeoutError included)
+        why = f"; hashlib pool unavailable: {type(exc).__name__}"
+    return {"value": wl.tokens_keyed() * passes / el, "unit": "tokens/s", "cores": cores,
             "kind": "oracle",
             "sample": f"{passes} full passes of the {wl.name} batch ({wl.batch.R} requests) in {el:.1f} s: "
-                      "C FIPS 180-4 SHA-256 (OpenMP over requests) + Python dict table"}
+                      "C FIPS 180-4 SHA-256 (OpenMP over requests) + Python dict table",
+            "keys_only_tokens_per_s": {
+                "c_one_thread": one, "c_all_cores": omp, "hashlib_processes": hl,
+                "sample": f"key derivation of the whole batch: C {n1} passes on 1 thread ({e1:.1f} s), {n2} on "
+                          f"{cores} threads ({e2:.1f} s); hashlib {n3} passes over {cores} spawned processes "
+                          f"({e3:.1f} s){why}"}}
+
+
+def critical_path(wl, derive_s: float, peaks: dict) -> dict:
+    """The serial bound of key derivation: a request's chain cannot start before its first chunk digest
+    and then takes 2 dependent compressions per chunk; a lone warp's compression cannot beat its
+    half-rate logic/shift pipe (10 such instructions per round, one every 2 cycles, 64 rounds)."""
+    C = wl.chunk_tokens
+    n_max = int((np.diff(wl.batch.tok_off) // C).max()) if wl.batch.R else 0
+    serial = (-(-(4 * C + 9) // 64) + 2 * n_max) if n_max else 0
+    per_comp_us = 64 * 10 * 2 / peaks["sm_max_mhz"]
+    bound_us = serial * per_comp_us
+    return {"serial_compressions": serial, "compression_floor_us": per_comp_us, "bound_us": bound_us,
+            "key_derivation_us": derive_s * 1e6, "frac": bound_us / (derive_s * 1e6) if derive_s else None,
+            "basis": "first chunk digest + 2 compressions per chunk of the longest request, each at least "
+                     "64 rounds x 10 logic/shift instructions x 2 cycles at the max SM clock"}
 
 
 def workload_config(wl, args) -> dict:
@@ -489,6 +548,7 @@ def main():
                                    "note": "all inputs read by the kernels from pinned host memory"}},
         # per step: chunk offsets, chunk+descriptor digests, chain; lookup-and-store (one kernel of
         # request warps, or per key + per-request tail for few long requests); finalize
+        "critical_path": critical_path(wl, derive_s, peaks),
         "gpu_launches": (3 + (1 if (R >= 1024 or N_cap <= 64 * R) else 2) + 1) * args.steps,
         "clocks": clk,
     }

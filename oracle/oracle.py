@@ -216,6 +216,33 @@ def derive_keys(tokens: np.ndarray, tok_off: np.ndarray, C: int, desc_idx: np.nd
     return key_off, keys[:N]
 
 
+def request_keys_hashlib(tokens: np.ndarray, C: int, d: bytes) -> np.ndarray:
+    """request_keys restated with the standard library's SHA-256 (OpenSSL):
+    c_i over the little-endian int32 bytes of chunk i, k_i = H(k_{i-1} || d || c_i)
+    from 32 zero bytes.  An independent second implementation of the chain,
+    and the CPU baseline that may use the host's SHA-2 instructions."""
+    import hashlib
+    raw = np.ascontiguousarray(tokens, dtype="<i4").tobytes()
+    n = len(raw) // (4 * C)
+    out = np.zeros((n, 32), np.uint8)
+    prev = bytes(32)
+    for i in range(n):
+        c = hashlib.sha256(raw[4 * C * i: 4 * C * (i + 1)]).digest()
+        prev = hashlib.sha256(prev + bytes(d) + c).digest()
+        out[i] = np.frombuffer(prev, np.uint8)
+    return out
+
+
+def derive_keys_hashlib(tokens: np.ndarray, tok_off: np.ndarray, C: int, desc_idx: np.ndarray,
+                        digests: np.ndarray, requests=None) -> np.ndarray:
+    """Keys of the given requests (default: all), concatenated, by request_keys_hashlib."""
+    tok_off = np.asarray(tok_off, np.int64)
+    digests = np.asarray(digests, np.uint8).reshape(-1, 32)
+    rows = [request_keys_hashlib(tokens[tok_off[r]:tok_off[r + 1]], C, digests[int(desc_idx[r])].tobytes())
+            for r in (range(tok_off.size - 1) if requests is None else requests)]
+    return np.concatenate(rows) if rows else np.zeros((0, 32), np.uint8)
+
+
 # --------------------------------------------------------------------------
 # Descriptor canonicalisation and enc (Sec. 5.2, 5.3)
 # --------------------------------------------------------------------------
