@@ -10,6 +10,8 @@
 // (pk_tensor_identity), so the tree is injective wherever SHA-256 is.
 #include <cuda_runtime.h>
 
+#include <mutex>
+
 #include "pk_device.cuh"
 #include "pk_internal.h"
 #include "pk_sha256.cuh"
@@ -65,9 +67,21 @@ struct TreeLevel {
 };
 static_assert(sizeof(TreeLevel) <= 4000, "kernel parameter space");
 
-__global__ void __launch_bounds__(kTreeThreads) k_tree_level(const TreeLevel lv) {
-    __shared__ uint32_t sK[64];
-    if (threadIdx.x < 64) sK[threadIdx.x] = pk::kSha256K[threadIdx.x];
+// K_t + W_t of the final block of every 1 KiB message: 0x80, zeros, the length in bits (8192).
+struct PadKW1K {
+    uint32_t kw[64];
+};
+
+// F is the round form of pk_sha256.cuh (kAddsFma for levels of many blocks);
+// `one` is its run-time constant 1.
+template <int F>
+__global__ void __launch_bounds__(kTreeThreads)
+k_tree_level(const __grid_constant__ TreeLevel lv, const __grid_constant__ PadKW1K pad, uint32_t one) {
+    __shared__ uint32_t sK[64], sPad[64];
+    if (threadIdx.x < 64) {
+        sK[threadIdx.x] = pk::kSha256K[threadIdx.x];
+        sPad[threadIdx.x] = pad.kw[threadIdx.x];
+    }
     __syncthreads();
     pk::pdl_wait();
     const uint64_t t = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -88,14 +102,9 @@ __global__ void __launch_bounds__(kTreeThreads) k_tree_level(const TreeLevel lv)
 #pragma unroll
             for (int k = 0; k < 16; ++k) w[k] = wn[k];
             if (q + 1 < kTreeBlock / 64) load_words(sg.src, sg.n, base + 64 * (q + 1), wn);
-            pk::compress_rolled(st, w, sK);
+            pk::compress_rolled<F>(st, w, sK, one);
         }
-        // padding of a 1024-byte message: 0x80, zeros, the length in bits (8192)
-#pragma unroll
-        for (int k = 0; k < 16; ++k) w[k] = 0;
-        w[0] = 0x80000000u;
-        w[15] = (uint32_t)(kTreeBlock * 8);
-        pk::compress_rolled(st, w, sK);
+        pk::compress_kw<F>(st, sPad, one);  // the padding block, rounds only
         uint4 *q = reinterpret_cast<uint4 *>(sg.dst + 32 * b);
         q[0] = make_uint4(pk::bswap32(st[0]), pk::bswap32(st[1]), pk::bswap32(st[2]), pk::bswap32(st[3]));
         q[1] = make_uint4(pk::bswap32(st[4]), pk::bswap32(st[5]), pk::bswap32(st[6]), pk::bswap32(st[7]));
@@ -104,6 +113,25 @@ __global__ void __launch_bounds__(kTreeThreads) k_tree_level(const TreeLevel lv)
 }
 
 uint64_t blocks_of(uint64_t n) { return n == 0 ? 1 : (n + kTreeBlock - 1) / kTreeBlock; }
+
+// Threads of a level from which the multiply-add round form is used (3 warps
+// per SM sub-partition, as for the chunk digests), computed once per device;
+// 0 (never) if the device cannot be queried.
+uint64_t fma_threshold() {
+    static std::mutex mu;
+    static uint64_t cache[256] = {};
+    static bool known[256] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return 0;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!known[dev]) {
+        int sms = 0;
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && sms > 0)
+            cache[dev] = 3ull * 4 * 32 * (uint64_t)sms;
+        known[dev] = true;
+    }
+    return cache[dev];
+}
 
 }  // namespace
 
@@ -122,6 +150,13 @@ uint64_t pk_content_scratch_bytes_impl(uint64_t n_bytes) {
 // levels go to scratch at scratch_off[j]; its last level writes tops[32 j].
 cudaError_t pk_launch_content_digests(const uint8_t *const *bytes, const uint64_t *n_bytes, uint32_t n,
                                       uint8_t *scratch, const uint64_t *scratch_off, uint8_t *tops, cudaStream_t s) {
+    PadKW1K pad;
+    {
+        const uint32_t m[16] = {0x80000000u, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, (uint32_t)(kTreeBlock * 8)};
+        pk::kw_table(m, pad.kw);
+    }
+    const uint64_t fma_from = fma_threshold();
+    const uint32_t one = 1u;
     for (uint32_t j0 = 0; j0 < n; j0 += kMaxSeg) {
         const uint32_t cnt = n - j0 < kMaxSeg ? n - j0 : kMaxSeg;
         TreeSeg cur[kMaxSeg];
@@ -147,8 +182,10 @@ cudaError_t pk_launch_content_digests(const uint8_t *const *bytes, const uint64_
             if (lv.count == 0) break;
             if (threads >= (1ull << 31)) return cudaErrorInvalidValue;
             lv.first[lv.count] = (uint32_t)threads;
-            const cudaError_t e =
-                pk_launch(k_tree_level, (unsigned)((threads + kTreeThreads - 1) / kTreeThreads), kTreeThreads, s, lv);
+            const unsigned grid = (unsigned)((threads + kTreeThreads - 1) / kTreeThreads);
+            const cudaError_t e = fma_from && threads >= fma_from
+                                      ? pk_launch(k_tree_level<pk::kAddsFma>, grid, kTreeThreads, s, lv, pad, one)
+                                      : pk_launch(k_tree_level<pk::kAddsPlain>, grid, kTreeThreads, s, lv, pad, one);
             if (e != cudaSuccess) return e;
             for (uint32_t j = 0; j < cnt; ++j) {  // the next level reads this one
                 if (done[j]) continue;

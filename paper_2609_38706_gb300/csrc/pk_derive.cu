@@ -183,12 +183,15 @@ __device__ __forceinline__ void load_tables(uint32_t *sK, uint32_t *sPad, const 
 // ---------------------------------------------------------------------------
 constexpr int kDigestBlock = 128;
 constexpr int kStages = 3;
+constexpr uint32_t kFmaWarps = 3;  // warps of chunks per SM sub-partition from which kAddsFma is used
 
-// c = SHA-256 of chunk g (request r), written to keys[g].
+// c = SHA-256 of chunk g (request r), written to keys[g].  F is the round
+// form (pk_sha256.cuh: kAddsFma when several warps share each sub-partition).
+template <int F>
 __device__ __forceinline__ void digest_chunk(const int32_t *tokens, const int64_t *tok_off,
                                              const int64_t *key_off, uint32_t r, int64_t g, uint32_t C,
                                              const uint32_t *sK, const uint32_t *sPad,
-                                             uint32_t (*ring)[kDigestBlock][16], uint8_t *keys) {
+                                             uint32_t (*ring)[kDigestBlock][16], uint8_t *keys, uint32_t one) {
     const int64_t i = g - __ldcg(key_off + r);
     const int32_t *src = tokens + __ldcg(tok_off + r) + i * (int64_t)C;
     const bool aligned = (reinterpret_cast<uintptr_t>(src) & 15) == 0;
@@ -218,20 +221,20 @@ __device__ __forceinline__ void digest_chunk(const int32_t *tokens, const int64_
                 w[4 * v + 2] = pk::bswap32(x.z);
                 w[4 * v + 3] = pk::bswap32(x.w);
             }
-            pk::compress_rolled(st, w, sK);
+            pk::compress_rolled<F>(st, w, sK, one);
         }
         cp_async_wait<0>();
     } else {
 #pragma unroll 1
         for (uint32_t b = 0; b < nfull; ++b) {
             load_block_global(src + 16 * b, w);
-            pk::compress_rolled(st, w, sK);
+            pk::compress_rolled<F>(st, w, sK, one);
         }
     }
     const uint64_t bits = (uint64_t)C * 32u;
     const int rem = (int)(C % 16);
     if (rem == 0) {
-        pk::compress_kw(st, sPad);
+        pk::compress_kw<F>(st, sPad, one);
     } else {
         const int32_t *tail = src + 16 * nfull;
 #pragma unroll
@@ -240,14 +243,14 @@ __device__ __forceinline__ void digest_chunk(const int32_t *tokens, const int64_
         if (rem <= 13) {
             w[14] = (uint32_t)(bits >> 32);
             w[15] = (uint32_t)bits;
-            pk::compress_rolled(st, w, sK);
+            pk::compress_rolled<F>(st, w, sK, one);
         } else {
-            pk::compress_rolled(st, w, sK);
+            pk::compress_rolled<F>(st, w, sK, one);
 #pragma unroll
             for (int t = 0; t < 16; ++t) w[t] = 0;
             w[14] = (uint32_t)(bits >> 32);
             w[15] = (uint32_t)bits;
-            pk::compress_rolled(st, w, sK);
+            pk::compress_rolled<F>(st, w, sK, one);
         }
     }
     store_digest(keys + 32 * g, st);
@@ -265,10 +268,12 @@ struct DescWork {
     uint32_t desc_blocks;
 };
 
+// `one` is the run-time constant 1 of the multiply-add round form.
+template <int F>
 __global__ void __launch_bounds__(kDigestBlock)
 k_chunk_digest(const int32_t *tokens, const int64_t *tok_off,
                const int64_t *key_off, uint32_t R, uint32_t C, const __grid_constant__ PadKW pad,
-               uint8_t *keys, const __grid_constant__ DescWork dw) {
+               uint8_t *keys, const __grid_constant__ DescWork dw, uint32_t one) {
     __shared__ uint32_t sK[64], sPad[64];
     __shared__ __align__(16) uint32_t ring[kStages][kDigestBlock][16];
     // The successor (the chain) is released as each block finishes, not at its start: released early,
@@ -299,7 +304,7 @@ k_chunk_digest(const int32_t *tokens, const int64_t *tok_off,
         const int64_t g0 = g - (threadIdx.x & 31);
         if (g0 >= g_end) break;  // whole warp past the end (uniform per warp)
         const uint32_t r = pk::lane_request(key_off, R, g0, g_end, g);
-        if (g < g_end) digest_chunk(tokens, tok_off, key_off, r, g, C, sK, sPad, ring, keys);
+        if (g < g_end) digest_chunk<F>(tokens, tok_off, key_off, r, g, C, sK, sPad, ring, keys, one);
         __syncwarp();
     }
     pk::pdl_launch_dependents();
@@ -524,14 +529,23 @@ cudaError_t pk_launch_derive_enc(const pk_ctx *ctx, const int32_t *tokens, uint6
     PadKW pad;
     for (int t = 0; t < 64; ++t) pad.kw[t] = ctx->pad_kw[t];
     const bool chunks = R > 0 && key_capacity > 0;
+    const uint32_t one = 1u;
     if (!chunks) {
         if (dw.desc_blocks)
-            e = pk_launch(k_chunk_digest, dw.desc_blocks, kDigestBlock, s, tokens, tok_off, (const int64_t *)key_off, 0u,
-                          C, pad, keys, dw);
+            e = pk_launch(k_chunk_digest<pk::kAddsPlain>, dw.desc_blocks, kDigestBlock, s, tokens, tok_off,
+                          (const int64_t *)key_off, 0u, C, pad, keys, dw, one);
         return e != cudaSuccess ? e : cudaGetLastError();
     }
-    e = pk_launch(k_chunk_digest, grid_for(key_capacity, kDigestBlock) + dw.desc_blocks, kDigestBlock, s, tokens,
-                  tok_off, (const int64_t *)key_off, R, C, pad, keys, dw);
+    // The multiply-add round form pays once at least kFmaWarps warps of chunks share each SM
+    // sub-partition (measured 10-13% per compression at 4 warps; slower for a lone warp).  The chunk
+    // count is at most key_capacity; with an unknown SM count the compiler's form is kept.
+    const uint64_t warps = (key_capacity + 31) / 32;
+    const bool fma = ctx->sm_count > 0 && warps >= (uint64_t)kFmaWarps * 4u * ctx->sm_count;
+    const unsigned grid = grid_for(key_capacity, kDigestBlock) + dw.desc_blocks;
+    e = fma ? pk_launch(k_chunk_digest<pk::kAddsFma>, grid, kDigestBlock, s, tokens, tok_off, (const int64_t *)key_off,
+                        R, C, pad, keys, dw, one)
+            : pk_launch(k_chunk_digest<pk::kAddsPlain>, grid, kDigestBlock, s, tokens, tok_off,
+                        (const int64_t *)key_off, R, C, pad, keys, dw, one);
     if (e != cudaSuccess) return e;
     e = pk_launch(k_chain, grid_for(R, kChainLanes), 2 * kChainLanes, s, (const int64_t *)key_off, desc_idx,
                   (const uint8_t *)digests, R, D, keys);

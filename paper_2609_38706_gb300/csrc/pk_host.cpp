@@ -170,6 +170,13 @@ int pk_init(pk_ctx **out, const pk_config *cfg, pk_stream stream) {
     c->table = static_cast<pk_entry *>(cfg->table_dev);
     c->epoch = 0;
     c->stamps = nullptr;
+    c->sm_count = 0;
+    {
+        int dev = 0, sms = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess &&
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && sms > 0)
+            c->sm_count = (uint32_t)sms;
+    }
     {   // final block of a 4C-byte message when 4C is a multiple of 64: 0x80, zeros, 64-bit bit length
         const uint64_t bits = (uint64_t)cfg->chunk_tokens * 32u;
         const uint32_t m[16] = {0x80000000u, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, 0, (uint32_t)(bits >> 32),

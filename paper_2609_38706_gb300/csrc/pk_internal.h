@@ -31,6 +31,7 @@ struct pk_ctx {
     unsigned long long epoch;         // last store call number
     unsigned long long *stamps;       // budget mode: last-use stamp per entry (pk_attach_stamps), else NULL
     uint32_t pad_kw[64];              // K_t + W_t of a chunk's final (padding-only) block, C % 16 == 0
+    uint32_t sm_count;                // SMs of the context's device (0 if unknown): picks the round form
 };
 
 // internal per-entry state between the two store kernels

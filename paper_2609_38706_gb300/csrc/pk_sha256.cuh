@@ -202,44 +202,96 @@ namespace pk {
 // working-variable rotation period 8 divides 16, so one body serves all four
 // quarters).  Keeping the code a quarter of the fully unrolled size keeps a
 // loop of several compressions resident in the instruction cache; the round
-// constants are read from a shared-memory copy (sK, 64 words, see load_k).
+// constants are read from a shared-memory copy (sK, 64 words) that each
+// kernel makes at its start.
+//
+// Pipes.  Every rotation, shift and 3-input logic operation of SHA-256 issues
+// on the SM's ALU pipe, one warp instruction per 2 cycles per sub-partition,
+// and so do the 3-input integer adds the compiler emits for most additions
+// (measured on GB300: SHF, LOP3 and IADD3 each 2.0 cycles per warp
+// instruction).  An integer multiply-add issues on the FMA pipe, at the same
+// rate and alongside the ALU (an SHF/IMAD pair: 2.1 cycles).  The two round
+// forms differ only in where the additions go, never in the value computed:
+//   kAddsPlain  the compiler's choice (ALU-bound at 25 cycles per round when
+//               the sub-partition is saturated, 29.8 for a lone warp);
+//   kAddsFma    every addition as x * one + y on the FMA pipe (`one` is a
+//               run-time 1 the compiler cannot fold): 22.2 cycles per round
+//               and 10-13% faster compressions once 4 or more warps share a
+//               sub-partition, but 33.4 cycles for a lone warp (the
+//               multiply-add's longer latency sits on the critical path).
+enum { kAddsPlain = 0, kAddsFma = 1 };
 
-__device__ __forceinline__ void round_kw(uint32_t &a, uint32_t &b, uint32_t &c, uint32_t &d, uint32_t &e,
-                                         uint32_t &f, uint32_t &g, uint32_t &h, uint32_t kw) {
-    const uint32_t t1 = h + big_s1(e) + ch(e, f, g) + kw;
-    const uint32_t t2 = big_s0(a) + maj(a, b, c);
-    h = g; g = f; f = e; e = d + t1; d = c; c = b; b = a; a = t1 + t2;
+// x * one + c, kept as a multiply-add (one == 1 at run time).
+__device__ __forceinline__ uint32_t mad1(uint32_t x, uint32_t one, uint32_t c) {
+    uint32_t r;
+    asm("mad.lo.u32 %0, %1, %2, %3;" : "=r"(r) : "r"(x), "r"(one), "r"(c));
+    return r;
 }
 
-template <bool SCHED>
-__device__ __forceinline__ void rounds16(uint32_t v[8], uint32_t w[16], const uint32_t *__restrict__ k16) {
+template <int F = kAddsPlain>
+__device__ __forceinline__ uint32_t add2(uint32_t x, uint32_t y, uint32_t one) {
+    if (F == kAddsFma) return mad1(x, one, y);
+    return x + y;
+}
+
+template <int F = kAddsPlain>
+__device__ __forceinline__ void round_kw(uint32_t &a, uint32_t &b, uint32_t &c, uint32_t &d, uint32_t &e,
+                                         uint32_t &f, uint32_t &g, uint32_t &h, uint32_t kw, uint32_t one = 1u) {
+    if (F == kAddsFma) {
+        const uint32_t t1 = mad1(big_s1(e), one, mad1(ch(e, f, g), one, mad1(h, one, kw)));
+        const uint32_t t2 = mad1(big_s0(a), one, maj(a, b, c));
+        h = g; g = f; f = e; e = mad1(d, one, t1); d = c; c = b; b = a; a = mad1(t1, one, t2);
+    } else {
+        const uint32_t t1 = h + big_s1(e) + ch(e, f, g) + kw;
+        const uint32_t t2 = big_s0(a) + maj(a, b, c);
+        h = g; g = f; f = e; e = d + t1; d = c; c = b; b = a; a = t1 + t2;
+    }
+}
+
+// W_t = s1(W_{t-2}) + W_{t-7} + s0(W_{t-15}) + W_{t-16} in the 16-word ring w, slot j.
+template <int F = kAddsPlain>
+__device__ __forceinline__ uint32_t sched_word(uint32_t w[16], int j, uint32_t one) {
+    if (F == kAddsFma)
+        w[j] = mad1(small_s1(w[(j + 14) & 15]), one,
+                    mad1(small_s0(w[(j + 1) & 15]), one, mad1(w[(j + 9) & 15], one, w[j])));
+    else
+        w[j] += small_s1(w[(j + 14) & 15]) + w[(j + 9) & 15] + small_s0(w[(j + 1) & 15]);
+    return w[j];
+}
+
+template <bool SCHED, int F = kAddsPlain>
+__device__ __forceinline__ void rounds16(uint32_t v[8], uint32_t w[16], const uint32_t *__restrict__ k16,
+                                         uint32_t one = 1u) {
     uint32_t a = v[0], b = v[1], c = v[2], d = v[3], e = v[4], f = v[5], g = v[6], h = v[7];
     uint32_t k[16];  // read before the first round, so that no round waits on shared memory
 #pragma unroll
     for (int j = 0; j < 16; ++j) k[j] = k16[j];
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
-        if (SCHED) w[j] += small_s1(w[(j + 14) & 15]) + w[(j + 9) & 15] + small_s0(w[(j + 1) & 15]);
-        round_kw(a, b, c, d, e, f, g, h, k[j] + w[j]);
+        if (SCHED) sched_word<F>(w, j, one);
+        round_kw<F>(a, b, c, d, e, f, g, h, add2<F>(k[j], w[j], one), one);
     }
     v[0] = a; v[1] = b; v[2] = c; v[3] = d; v[4] = e; v[5] = f; v[6] = g; v[7] = h;
 }
 
 // st <- st + compress(st, w); w is overwritten by the schedule.
-__device__ __forceinline__ void compress_rolled(uint32_t st[8], uint32_t w[16], const uint32_t *__restrict__ sK) {
+template <int F = kAddsPlain>
+__device__ __forceinline__ void compress_rolled(uint32_t st[8], uint32_t w[16], const uint32_t *__restrict__ sK,
+                                                uint32_t one = 1u) {
     uint32_t v[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) v[j] = st[j];
-    rounds16<false>(v, w, sK);
+    rounds16<false, F>(v, w, sK, one);
 #pragma unroll 1
-    for (int q = 1; q < 4; ++q) rounds16<true>(v, w, sK + 16 * q);
+    for (int q = 1; q < 4; ++q) rounds16<true, F>(v, w, sK + 16 * q, one);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) st[j] += v[j];
+    for (int j = 0; j < 8; ++j) st[j] = add2<F>(st[j], v[j], one);
 }
 
 // st <- st + compress(st, W) for a message whose whole schedule is known in
 // advance: kw[t] = K_t + W_t for t = 0..63 (rounds only).
-__device__ __forceinline__ void compress_kw(uint32_t st[8], const uint32_t *__restrict__ kw) {
+template <int F = kAddsPlain>
+__device__ __forceinline__ void compress_kw(uint32_t st[8], const uint32_t *__restrict__ kw, uint32_t one = 1u) {
     uint32_t a = st[0], b = st[1], c = st[2], d = st[3], e = st[4], f = st[5], g = st[6], h = st[7];
 #pragma unroll 1
     for (int q = 0; q < 4; ++q) {
@@ -247,9 +299,11 @@ __device__ __forceinline__ void compress_kw(uint32_t st[8], const uint32_t *__re
 #pragma unroll
         for (int j = 0; j < 16; ++j) x[j] = kw[16 * q + j];
 #pragma unroll
-        for (int j = 0; j < 16; ++j) round_kw(a, b, c, d, e, f, g, h, x[j]);
+        for (int j = 0; j < 16; ++j) round_kw<F>(a, b, c, d, e, f, g, h, x[j], one);
     }
-    st[0] += a; st[1] += b; st[2] += c; st[3] += d; st[4] += e; st[5] += f; st[6] += g; st[7] += h;
+    st[0] = add2<F>(st[0], a, one); st[1] = add2<F>(st[1], b, one); st[2] = add2<F>(st[2], c, one);
+    st[3] = add2<F>(st[3], d, one); st[4] = add2<F>(st[4], e, one); st[5] = add2<F>(st[5], f, one);
+    st[6] = add2<F>(st[6], g, one); st[7] = add2<F>(st[7], h, one);
 }
 
 }  // namespace pk

@@ -39,6 +39,13 @@ def test_large_buffer_against_the_oracle():
     assert gpu_top(data) == O.content_digest(data.tobytes())
 
 
+def test_level_of_many_blocks_against_the_oracle():
+    """96 MiB: a first tree level of 98,305 blocks, enough warps per SM sub-partition for the multiply-add
+    round form (every addition on the FMA pipe), bit-exact like the compiler's form."""
+    data = np.random.default_rng(96).integers(0, 256, 96 * (1 << 20) + 5, dtype=np.uint8)
+    assert gpu_top(data) == O.content_digest(data.tobytes())
+
+
 def test_adapter_identity_end_to_end():
     from paper_2609_38706_gb300 import pk
     rng = np.random.default_rng(8)
