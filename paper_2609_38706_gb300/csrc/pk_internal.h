@@ -27,7 +27,7 @@ struct pk_ctx {
     uint32_t max_probe;
     uint64_t capacity;
     pk_entry *table;
-    unsigned long long *counter_dev;  // number of entries in the table
+    unsigned long long *counter_dev;  // [0] entries in the table; [1] requests handed out by a lookup-and-store
     unsigned long long epoch;         // last store call number
     unsigned long long *stamps;       // budget mode: last-use stamp per entry (pk_attach_stamps), else NULL
     uint32_t pad_kw[64];              // K_t + W_t of a chunk's final (padding-only) block, C % 16 == 0

@@ -760,18 +760,15 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
 // ends with PK_ERR_ARG when it lies in the store range.
 // ---------------------------------------------------------------------------
 
-// One warp per request, refilled from a register buffer as k_lookup_req.
-__global__ void __launch_bounds__(256, 3)
-k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
-                   unsigned long long *counter, unsigned long long epoch, unsigned long long *stamps, const uint8_t *keys,
-                   const uint32_t *new_slots, const int64_t *key_off, uint32_t R,
-                   uint64_t key_capacity, uint32_t *slots, int32_t *hit,
-                   int32_t *result, uint32_t *slot_out, int32_t *status) {
-    __shared__ unsigned long long block_claims;
-    if (threadIdx.x == 0) block_claims = 0;
-    __syncthreads();
-    pk::pdl_wait(table, counter, keys, new_slots, key_off, slots, hit, result, slot_out, status);
-    const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+// One request r (warp-uniform; r >= R does nothing), refilled from a register
+// buffer as k_lookup_req.  `release`: release the finalize launch after the
+// probes (the kernel with one request per warp).
+__device__ __forceinline__ void lookup_store_request(const ClaimCtx &c, uint64_t r, const uint8_t *keys,
+                                                     const uint32_t *new_slots, const int64_t *key_off, uint32_t R,
+                                                     uint64_t key_capacity, uint32_t *slots, int32_t *hit,
+                                                     int32_t *result, uint32_t *slot_out, int32_t *status,
+                                                     uint32_t &claims, bool release) {
+    const uint64_t mask = c.mask;
     const uint32_t lane = threadIdx.x & 31;
     int64_t a = 0, b = 0;
     if (r < R) {  // uniform per warp
@@ -779,11 +776,6 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
         b = __ldcg(key_off + r + 1);
         if ((uint64_t)b > key_capacity) b = (int64_t)key_capacity;
     }
-    unsigned long long cnt = 0;
-    if (lane == 0) cnt = ld_volatile_u64(counter);
-    const bool fast = __shfl_sync(kFull, cnt, 0) + key_capacity < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast, stamps};
-    uint32_t claims = 0;
     uint32_t first_miss = 0xffffffffu;  // lowest miss index (relative to a) seen by this lane
     int64_t arg_hit = -1;               // highest index of a hit whose slot was PK_NO_SLOT
     ProbeKey s;
@@ -842,7 +834,7 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
             }
         }
     }
-    pk::pdl_launch_dependents();  // main work done: release the finalize kernel
+    if (release) pk::pdl_launch_dependents();  // main work done: release the finalize kernel
     const uint32_t hm = __reduce_min_sync(kFull, first_miss);
     const int64_t h = hm != 0xffffffffu ? (int64_t)hm : (b > a ? b - a : 0);
     __syncwarp();
@@ -852,6 +844,47 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
     }
     if (r < R && lane == 0) hit[r] = (int32_t)h;
     if (arg_hit >= a + h) set_status(status, PK_ERR_ARG);
+}
+
+// Next request for a work-taking warp: tickets[0] counts the requests handed
+// out in this call (zeroed before the launch).
+__device__ __forceinline__ uint64_t take_request(unsigned long long *tickets) {
+    unsigned long long t = 0;
+    if ((threadIdx.x & 31) == 0) t = atomicAdd(tickets, 1ull);
+    return __shfl_sync(kFull, t, 0);
+}
+
+// One warp per request (kTake false: warp w serves request w), or a grid of
+// resident CTAs whose warps take requests one at a time until none is left
+// (kTake true, for batches of more requests than resident warps: a warp done
+// with its request does not wait for the slowest request of its block).
+template <bool kTake>
+__global__ void __launch_bounds__(256, 3)
+k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
+                   unsigned long long *counter, unsigned long long epoch, unsigned long long *stamps, const uint8_t *keys,
+                   const uint32_t *new_slots, const int64_t *key_off, uint32_t R,
+                   uint64_t key_capacity, uint32_t *slots, int32_t *hit,
+                   int32_t *result, uint32_t *slot_out, int32_t *status, unsigned long long *tickets) {
+    __shared__ unsigned long long block_claims;
+    if (threadIdx.x == 0) block_claims = 0;
+    __syncthreads();
+    pk::pdl_wait(table, counter, keys, new_slots, key_off, slots, hit, result, slot_out, status, tickets);
+    const uint32_t lane = threadIdx.x & 31;
+    unsigned long long cnt = 0;
+    if (lane == 0) cnt = ld_volatile_u64(counter);
+    const bool fast = __shfl_sync(kFull, cnt, 0) + key_capacity < capacity;
+    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast, stamps};
+    uint32_t claims = 0;
+    if (kTake) {
+        for (uint64_t r = take_request(tickets); r < R; r = take_request(tickets))
+            lookup_store_request(c, r, keys, new_slots, key_off, R, key_capacity, slots, hit, result, slot_out,
+                                 status, claims, false);
+        pk::pdl_launch_dependents();
+    } else {
+        const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+        lookup_store_request(c, r, keys, new_slots, key_off, R, key_capacity, slots, hit, result, slot_out, status,
+                             claims, true);
+    }
     count_claims(&block_claims, claims, counter);
 }
 
@@ -1091,6 +1124,27 @@ unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1
 // walk them serially).
 bool per_request(uint32_t R, uint64_t key_capacity) { return R >= 1024 || key_capacity <= 64ull * R; }
 
+// Resident CTAs of k_lookup_store_req (SMs x CTAs per SM) on the current
+// device, computed once per device.
+cudaError_t lookup_store_resident(uint64_t *out) {
+    static std::mutex mu;
+    static uint64_t cache[256] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 256) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!cache[dev]) {
+        int sms = 0, per_sm = 0;
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_lookup_store_req<true>, 256, 0);
+        if (e != cudaSuccess) return e;
+        cache[dev] = (uint64_t)sms * (uint64_t)(per_sm < 1 ? 1 : per_sm);
+    }
+    *out = cache[dev];
+    return cudaSuccess;
+}
+
 }  // namespace
 
 cudaError_t pk_launch_load_table(const pk_ctx *ctx, const void *src, cudaStream_t s) {
@@ -1158,9 +1212,21 @@ cudaError_t pk_launch_lookup_store(const pk_ctx *ctx, unsigned long long epoch, 
     const uint64_t mask = ctx->capacity - 1;
     cudaError_t e;
     if (per_request(R, key_capacity)) {
-        e = pk_launch(k_lookup_store_req, grid_for(32ull * R, 256), 256, s, ctx->table, mask, ctx->max_probe,
-                      ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, new_slots, key_off, R, key_capacity, slots,
-                      hit_chunks, result, slot_out, status);
+        uint64_t resident = 0;
+        e = lookup_store_resident(&resident);
+        if (e != cudaSuccess) return e;
+        unsigned long long *tickets = ctx->counter_dev + 1;
+        if (R > 32 * resident) {  // more requests than resident warps: warps take requests as they finish
+            e = cudaMemsetAsync(tickets, 0, sizeof *tickets, s);
+            if (e == cudaSuccess)
+                e = pk_launch(k_lookup_store_req<true>, (unsigned)resident, 256, s, ctx->table, mask, ctx->max_probe,
+                              ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, new_slots, key_off, R,
+                              key_capacity, slots, hit_chunks, result, slot_out, status, tickets);
+        } else {
+            e = pk_launch(k_lookup_store_req<false>, grid_for(32ull * R, 256), 256, s, ctx->table, mask,
+                          ctx->max_probe, ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, new_slots, key_off,
+                          R, key_capacity, slots, hit_chunks, result, slot_out, status, tickets);
+        }
     } else {
         e = key_capacity == 0
                 ? cudaSuccess

@@ -124,16 +124,19 @@ def _rows(rng, R, C, lo, hi):
             for _ in range(R)]
 
 
-@pytest.mark.parametrize("shape", ["many_short", "few_long"])
+@pytest.mark.parametrize("shape", ["many_short", "few_long", "more_requests_than_warps"])
 def test_reserved_slots_zero_keys_and_empty_requests(shape):
     """Keys whose new slot is PK_NO_SLOT (in the hit prefix: skipped; in the
     miss range: PK_ERR_ARG), all-zero keys, empty requests, duplicates across
-    requests; both the per-request path (many short requests) and the
-    per-key path (few long requests)."""
+    requests; the per-request path (many short requests), the per-key path
+    (few long requests), and the per-request path with more requests than
+    resident warps (warps take requests as they finish: 30,000 requests
+    against 152 SMs x 3 CTAs x 8 warps on GB300)."""
     from paper_2609_38706_gb300.service import KeyTable, u32
-    rng = np.random.default_rng(7 if shape == "many_short" else 8)
+    rng = np.random.default_rng({"many_short": 7, "few_long": 8, "more_requests_than_warps": 9}[shape])
     C = 16
-    R, lo, hi = (1500, 0, 6) if shape == "many_short" else (3, 200, 400)
+    R, lo, hi = {"many_short": (1500, 0, 6), "few_long": (3, 200, 400),
+                 "more_requests_than_warps": (30_000, 0, 6)}[shape]
     rows = _rows(rng, R, C, lo, hi)
     for r in range(1, R, 3):  # shared prefixes: duplicate keys across requests
         n = min(len(rows[r]), len(rows[r - 1]))
@@ -155,7 +158,7 @@ def test_reserved_slots_zero_keys_and_empty_requests(shape):
     seed_idx = seed_idx[~np.isin(seed_idx, zero_at)]
     new_slots = np.arange(N, dtype=np.uint32) + 5000
     new_slots[rng.choice(N, size=max(1, N // 50), replace=False)] = O.NO_SLOT
-    log2 = 14
+    log2 = 14 if shape != "more_requests_than_warps" else 17
     t = O.DictTable(1 << log2)
     t.store(keys[seed_idx], seed_idx.astype(np.uint32))
     hit, slots = O.lookup(t, keys, ko)
