@@ -144,6 +144,54 @@ def test_budget_mode_stamps():
     kt.close()
 
 
+def test_budget_mode_stamps_with_more_requests_than_warps():
+    """Stamps raised by pk_lookup_store when its warps take requests from a
+    counter (30,000 short requests against 152 SMs x 3 CTAs x 8 warps on
+    GB300): which warp serves a request must not change any stamp, slot or
+    result, so they equal the oracle's budget table."""
+    from paper_2609_38706_gb300.service import KeyTable, u32
+    rng = np.random.default_rng(31)
+    C, R = 16, 30_000
+    rows = [rng.integers(0, 40_000, int(rng.integers(0, 6)) * C, dtype=np.int64).astype(np.int32) for _ in range(R)]
+    for r in range(1, R, 3):  # shared prefixes: the same keys in several requests
+        n = min(len(rows[r]), len(rows[r - 1]))
+        rows[r][: n // 2] = rows[r - 1][: n // 2]
+    toks = np.concatenate(rows)
+    off = np.zeros(R + 1, np.int64)
+    np.cumsum([len(x) for x in rows], out=off[1:])
+    desc = [{"model_id": "m", "weight_precision": "bf16", "weight_version": "v", "adapter_id": "",
+             "kv_format": "bf16", "salt": ""}]
+    ko, keys = O.derive_keys(toks, off, C, np.zeros(R, np.uint32), O.descriptor_digests(desc))
+    N = keys.shape[0]
+    seed_idx = np.concatenate([np.arange(ko[r], ko[r] + (ko[r + 1] - ko[r]) // 2) for r in range(0, R, 2)])
+    log2 = 17
+    kt = KeyTable(C, log2)
+    kt.attach_stamps()
+    kt.store(torch.from_numpy(keys[seed_idx]).cuda(), seed_idx.astype(np.uint32))
+    kt.check("seed")
+    bt = O.BudgetTable(1 << log2)
+    bt.store(keys[seed_idx], seed_idx.astype(np.uint32))
+    new_slots = np.arange(N, dtype=np.uint32) + 5_000_000
+    hit, slots, res, so = kt.lookup_store(torch.from_numpy(keys).cuda(), torch.from_numpy(ko).cuda(), new_slots)
+    kt.check("lookup_store")
+    t = O.DictTable(1 << log2)
+    t.store(keys[seed_idx], seed_idx.astype(np.uint32))
+    r_hit, r_slots = O.lookup(t, keys, ko)
+    r_res, r_so = O.store_misses(t, keys, ko, r_hit, new_slots)
+    assert np.array_equal(hit.cpu().numpy(), r_hit)
+    assert np.array_equal(u32(slots), r_slots)
+    assert np.array_equal(res.cpu().numpy(), r_res)
+    assert np.array_equal(u32(so), r_so)
+    bt.lookup_store(keys, ko, new_slots)
+    e = kt.table.view(-1, 32).cpu().numpy()
+    st = kt.stamps.cpu().numpy().view(np.uint64)
+    occ = e[:, :16].any(axis=1)
+    tslots = e[:, 16:20].copy().view(np.uint32)[:, 0]
+    got = sorted(zip((bytes(k) for k in e[occ, :16]), tslots[occ].tolist(), st[occ].tolist()))
+    assert got == bt.triples()
+    kt.close()
+
+
 @pytest.mark.parametrize("shape", ["empty_batch", "no_full_chunks", "mixed"])
 def test_empty_and_short_requests(shape):
     from paper_2609_38706_gb300.service import KeyTable, u32
