@@ -408,11 +408,10 @@ int pk_table_load(pk_ctx *ctx, const void *src, size_t src_bytes, pk_stream stre
 
 /* Device.  The insert-if-absent of pk_store for callers that cannot allocate
  * device memory and so cannot create a context (pk_init allocates the
- * context's entry counter): code that runs while a CUDA graph is being
- * captured, engines whose device memory is entirely owned by their own pool
- * with a fixed budget, and latency-critical paths that must not enter the
- * CUDA allocator.  The paper has no counterpart; this is an integration
- * convenience.
+ * context's entry counter): engines whose device memory is entirely owned by
+ * their own pool with a fixed budget, and latency-critical paths that must
+ * not enter the CUDA allocator (an allocation can synchronise the device).
+ * The paper has no counterpart; this is an integration convenience.
  * The table is described by cfg (table_dev, table_bytes, capacity_log2,
  * max_probe; chunk_tokens is ignored) and must be all zero before its first
  * use (cudaMemset, or a table created by pk_init).  Arguments, results and

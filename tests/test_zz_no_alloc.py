@@ -1,8 +1,8 @@
 """GPU test of pk_store_noalloc, the store entry point that allocates nothing.
 
-Callers that cannot allocate device memory (code running while a CUDA graph
-is captured, engines whose device memory belongs to their own fixed pool,
-allocator-free latency paths) cannot create a libpk context, because pk_init
+Callers that cannot allocate device memory (engines whose device memory
+belongs to their own fixed pool, latency-critical paths that must stay out of
+the CUDA allocator) cannot create a libpk context, because pk_init
 allocates the context's entry counter.  pk_store_noalloc serves them: it keeps
 its scratch in a fixed device array inside the library.  Its results must be
 those of pk_store (the context entry point) on the same inputs, call after
