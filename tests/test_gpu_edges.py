@@ -51,6 +51,25 @@ def test_chunk_sizes_and_unaligned_starts(C):
     kt.close()
 
 
+@pytest.mark.parametrize("C", [21, 30])
+def test_multiply_add_round_form_with_ragged_unaligned_requests(C):
+    """A batch of more than 3 x 4 x 32 x 152 = 58,368 chunks, so that the
+    chunk digests run in the multiply-add round form, with requests of random
+    token counts (unaligned starts: 16-byte token loads and plain loads), and
+    chunk sizes whose final block holds tokens and the padding (C = 21, 5
+    tokens and the length in one block) or spills the length into a second
+    padding block (C = 30, 14 tokens)."""
+    rng = np.random.default_rng(1000 + C)
+    R = 6000
+    rows = [rng.integers(-2**31, 2**31, int(rng.integers(0, 40 * C)), dtype=np.int64).astype(np.int32)
+            for _ in range(R)]
+    assert sum(len(r) // C for r in rows) > 58_368
+    kt = KT(C)
+    ko, keys, rko, rkeys = derive_both(kt, rows, rng.integers(0, 2, R), [DESC, dict(DESC, adapter_id="a1")], C)
+    assert np.array_equal(ko, rko) and np.array_equal(keys, rkeys)
+    kt.close()
+
+
 def test_published_vector_chunks():
     # FIPS 180-2 B.3 message (10^6 'a') as one 250000-token chunk, and B.2 as one 14-token chunk.
     a = np.full(250000, 0x61616161, np.int32)
