@@ -125,3 +125,95 @@ def test_load_zeroes_attached_stamps():
     assert not kt.stamps.any()
     assert kt.entries() == 300
     kt.close()
+
+
+_SEEDER = r'''
+import sys
+import numpy as np
+import torch
+sys.path.insert(0, sys.argv[1])
+import __graft_entry__ as g
+g.build()
+from paper_2609_38706_gb300 import workloads as W
+from paper_2609_38706_gb300.service import KeyTable
+wl = W.reduced("multi_adapter")
+b = wl.batch
+kt = KeyTable(wl.chunk_tokens, wl.capacity_log2)
+d = kt.digests(wl.descriptors)
+key_off, keys = kt.derive(b.tokens, b.tok_off, b.desc_idx, d)
+N = int(key_off[-1])
+kt.store(keys[:N], np.arange(N, dtype=np.uint32) + 7000)
+kt.check("seeder")
+snap = torch.empty(kt.table.numel() + 64, dtype=torch.uint8).pin_memory()
+kt.save(snap)
+torch.cuda.synchronize()
+np.save(sys.argv[2], snap.numpy())
+'''
+
+
+def test_seeder_and_retriever_in_separate_processes(tmp_path):
+    """The paper's two-phase setup: a seeder process derives a batch's keys,
+    stores them and saves the table; a retriever process loads the table and
+    derives the keys again on its own.  Every request then hits in full with
+    the seeder's slots, as the oracle's store-then-lookup says, and the same
+    tokens under another salt hit nothing."""
+    import os
+    import subprocess
+    import sys
+    from paper_2609_38706_gb300.service import KeyTable, u32
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    path = str(tmp_path / "table.npy")
+    subprocess.run([sys.executable, "-c", _SEEDER, root, path], check=True, timeout=600)
+    wl = W.reduced("multi_adapter")
+    b = wl.batch
+    kt = KeyTable(wl.chunk_tokens, wl.capacity_log2)
+    kt.load(torch.from_numpy(np.load(path)).pin_memory())
+    d = kt.digests(wl.descriptors)
+    key_off, keys = kt.derive(b.tokens, b.tok_off, b.desc_idx, d)
+    hit, slots = kt.lookup(keys, key_off)
+    kt.check("retriever")
+    ko = key_off.cpu().numpy()
+    N = int(ko[-1])
+    dd = O.descriptor_digests(wl.descriptors)
+    rko, rkeys = O.derive_keys(b.tokens, b.tok_off, wl.chunk_tokens, b.desc_idx, dd)
+    t = O.DictTable(wl.capacity)
+    t.store(rkeys, np.arange(N, dtype=np.uint32) + 7000)
+    rhit, rslots = O.lookup(t, rkeys, rko)
+    assert np.array_equal(ko, rko)
+    assert np.array_equal(hit.cpu().numpy(), rhit) and np.array_equal(rhit, np.diff(rko))
+    assert np.array_equal(u32(slots)[:N], rslots)
+    other = [dict(x, salt="another-domain") for x in wl.descriptors]
+    ko2, keys2 = kt.derive(b.tokens, b.tok_off, b.desc_idx, kt.digests(other))
+    hit2, _ = kt.lookup(keys2, ko2)
+    kt.check("retriever, other salt")
+    assert not hit2.cpu().numpy().any()
+    kt.close()
+
+
+def test_seeded_table_is_a_linear_probing_layout():
+    """The device table is plain linear probing from the home entry (the first 8 key bytes, little-endian,
+    modulo the capacity): every stored key lies at or after its home with no empty entry in between, and the
+    mean successful probe length of the seeded multi-adapter table (2^20 entries at load 0.5) is Knuth's
+    (1 + 1/(1 - a)) / 2 = 1.5 within 3% (a sanity check of the layout; results never depend on it)."""
+    wl = W.FULL_CONFIGS["multi_adapter"]()
+    kt, _ = _seeded(wl)
+    e = kt.table.view(-1, 32).cpu().numpy()
+    kt.close()
+    cap = e.shape[0]
+    mask = cap - 1
+    occ = e[:, :16].any(axis=1)
+    n = int(occ.sum())
+    assert n == wl.target_entries
+    home = e[:, :8].copy().view("<u8")[:, 0] & np.uint64(mask)
+    dist = (np.arange(cap, dtype=np.uint64) - home) & np.uint64(mask)
+    # length of the run of occupied entries ending at each entry, on a rotation that starts after an empty one
+    shift = int(np.flatnonzero(~occ)[0]) + 1
+    r = np.roll(occ, -shift)
+    idx = np.arange(cap)
+    last_empty = np.maximum.accumulate(np.where(~r, idx, -1))
+    run = np.roll(idx - last_empty, shift)
+    assert np.all(dist[occ] < run[occ].astype(np.uint64)), "a key is not reachable from its home"
+    alpha = n / cap
+    mean = float((dist[occ] + 1).mean())
+    knuth = 0.5 * (1 + 1 / (1 - alpha))
+    assert abs(mean - knuth) / knuth < 0.03, (mean, knuth)
