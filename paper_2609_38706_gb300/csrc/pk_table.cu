@@ -1159,7 +1159,8 @@ cudaError_t pk_launch_load_table(const pk_ctx *ctx, const void *src, cudaStream_
 
 cudaError_t pk_launch_mark_loaded(const pk_ctx *ctx, cudaStream_t s) {
     const uint64_t blocks = (ctx->capacity + 255) / 256;
-    k_mark_loaded<<<(unsigned)(blocks < 152 * 16 ? blocks : 152 * 16), 256, 0, s>>>(ctx->table, ctx->capacity);
+    const uint64_t cap = ctx->sm_count ? 16ull * ctx->sm_count : blocks;  // grid-strided: any grid is correct
+    k_mark_loaded<<<(unsigned)(blocks < cap ? blocks : cap), 256, 0, s>>>(ctx->table, ctx->capacity);
     return cudaGetLastError();
 }
 
@@ -1258,6 +1259,22 @@ static void *noalloc_scratch_addr(int device) {
     return addr[device];
 }
 
+// SMs of a device (0 if the query fails), queried once per device.
+static uint32_t device_sms(int device) {
+    static std::mutex mu;
+    static uint32_t sms[256] = {};
+    static bool known[256] = {};
+    if (device < 0 || device >= 256) return 0;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!known[device]) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, device) == cudaSuccess && n > 0)
+            sms[device] = (uint32_t)n;
+        known[device] = true;
+    }
+    return sms[device];
+}
+
 cudaError_t pk_launch_store_noalloc(pk_entry *table, uint32_t capacity_log2, uint32_t max_probe,
                                     const uint8_t *keys, const uint32_t *slots, uint64_t n, const int64_t *key_off,
                                     const int32_t *hit_chunks, uint32_t R, int32_t *result, uint32_t *slot_out,
@@ -1273,7 +1290,9 @@ cudaError_t pk_launch_store_noalloc(pk_entry *table, uint32_t capacity_log2, uin
     e = cudaMemsetAsync(sc, 0, 2 * sizeof(unsigned long long), s);
     if (e != cudaSuccess) return e;
     const uint64_t scan_blocks = (capacity + 255) / 256;
-    k_noalloc_scan<<<(unsigned)(scan_blocks < 152 * 8 ? scan_blocks : 152 * 8), 256, 0, s>>>(table, capacity, sc);
+    const uint32_t sms = device_sms(device);
+    const uint64_t scan_cap = sms ? 8ull * sms : scan_blocks;  // grid-strided: any grid is correct
+    k_noalloc_scan<<<(unsigned)(scan_blocks < scan_cap ? scan_blocks : scan_cap), 256, 0, s>>>(table, capacity, sc);
     k_noalloc_claim<<<grid_for(n, 256), 256, 0, s>>>(table, capacity - 1, max_probe, capacity, sc, keys, slots, n,
                                                       key_off, hit_chunks, key_off ? R : 0, result, slot_out, status);
     k_noalloc_finalize<<<grid_for(n, 256), 256, 0, s>>>(table, sc, n, result, slot_out);
