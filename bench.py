@@ -7,8 +7,10 @@ One step = one pass of the whole hot path over one batch:
   a1  chunk digests c_i          a2  chained keys k_i
   a3  probe every key            a4  store the miss ranges
 (a3 and a4 in one pass: pk_lookup_store).
-Default workload: the multi-adapter serving configuration (1024 requests x
-4096 tokens, chunk 256, 32 descriptors, table of 2^20 entries at load 0.5).
+Default workload: the small-block paged-cache configuration, the largest
+single-GPU one (16384 requests x 2048 tokens, chunk 16, 16 descriptors, table
+of 2^23 entries at load 0.6).  Without --steps, the number of timed steps is
+chosen from the warm-up so that the timed region lasts at least a second.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the CPU oracle on the same workload
@@ -39,8 +41,9 @@ sys.path.insert(0, ROOT)
 
 METRIC = "tokens keyed+looked up/sec and % of SHA-256/HBM roofline (1 GB300)"
 SHA_OPS_PER_COMPRESSION = 1384      # 64 rounds x 14 + 48 schedule words x 10 + 8 feed-forward
-SMS, LANES_PER_SM = 152, 128        # 4 SM sub-partitions x 32 lanes, one instruction each per clock
+LANES_PER_SM = 128                  # 4 SM sub-partitions x 32 lanes, one instruction each per clock
 L2_FLUSH_BYTES = 256 << 20
+MIN_TIMED_S = 1.2                   # default timed region: long enough for several clock samples
 
 
 def load_peaks():
@@ -58,8 +61,8 @@ DERIVE_SOURCES = ("paper_2609_38706_gb300/csrc/pk_derive.cu", "paper_2609_38706_
 
 def derive_traffic(workload: str):
     """Cold-cache DRAM bytes of one key-derivation call, from the committed ncu
-    summary, or None when the kernels changed since it was taken (or another
-    workload is run)."""
+    summary of that workload (profiles/dram_traffic_<workload>.md), or None
+    when there is none or the kernels changed since it was taken."""
     import hashlib
     h = hashlib.sha256()
     for f in DERIVE_SOURCES:
@@ -67,7 +70,7 @@ def derive_traffic(workload: str):
             h.update(fh.read())
     fields = {}
     try:
-        with open(os.path.join(ROOT, "profiles", "dram_traffic_multi_adapter.md")) as fh:
+        with open(os.path.join(ROOT, "profiles", f"dram_traffic_{workload}.md")) as fh:
             for line in fh:
                 k, _, v = line.strip().partition(":")
                 if v:
@@ -221,6 +224,14 @@ def run_cpu_baseline(wl, seconds: float) -> dict:
                           f"({e3:.1f} s){why}"}}
 
 
+def auto_steps(iter_s: float, min_s: float = MIN_TIMED_S, lo: int = 20, hi: int = 4000) -> int:
+    """Timed steps for a timed region of at least min_s, given the wall time
+    of one step with its untimed preparation."""
+    if iter_s <= 0:
+        return lo
+    return int(min(hi, max(lo, -(-min_s // iter_s))))
+
+
 def critical_path(wl, derive_s: float, peaks: dict) -> dict:
     """The serial bound of key derivation: a request's chain cannot start before its first chunk digest
     and then takes 2 dependent compressions per chunk; a lone warp's compression cannot beat its
@@ -292,10 +303,10 @@ def run_reference(args, rank: int, world: int) -> None:
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=0, help="timed steps (default: a timed region of >= 1.2 s)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="pk", choices=["pk", "reference"])
-    ap.add_argument("--workload", default="multi_adapter")
+    ap.add_argument("--workload", default="small_block")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
@@ -307,6 +318,8 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
 
     if args.impl == "reference":
+        if args.steps <= 0:
+            args.steps = 3
         run_reference(args, rank, world)
         return
 
@@ -321,6 +334,7 @@ def main():
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
     torch.cuda.set_stream(torch.cuda.Stream(device=dev))  # a dedicated (non-legacy) stream for all work
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
@@ -405,10 +419,15 @@ def main():
     n_keys = wl.n_keys()
 
     # ---- warm-up, then timed device-resident steps ----
+    t_warm = time.perf_counter()
     for _ in range(args.warmup):
         between_steps()
+        torch.cuda._sleep(spin_cycles)
         core()
-    torch.cuda.synchronize()
+        torch.cuda.synchronize()
+    iter_s = (time.perf_counter() - t_warm) / args.warmup
+    if args.steps <= 0:  # a timed region of at least MIN_TIMED_S, the same on every rank
+        args.steps = int(max_over_ranks([auto_steps(iter_s)], world, dev)[0])
     if kt.take_status() != 0:
         raise RuntimeError("device status after warm-up")
     hit_ref = hit_d.cpu().numpy().copy()
@@ -500,11 +519,11 @@ def main():
     peaks = load_peaks()
     c_dig, c_chain = compressions(n_keys, C)
     derive_s = float(np.mean(derive_ms)) / 1e3
-    alu_peak = SMS * LANES_PER_SM * peaks["sm_max_mhz"] * 1e6 / 1e12           # Tops/s, issue-rate ceiling
+    alu_peak = sms * LANES_PER_SM * peaks["sm_max_mhz"] * 1e6 / 1e12           # Tops/s, issue-rate ceiling
     # the logic/shift pipe takes 16 lanes per sub-partition per clock and SHA-256 with funnel-shift
     # rotations needs 1024 of its operations per compression (6 SHF + 4 LOP3 per round, 6 + 2 per
     # schedule word): the ceiling for this formulation, in the same 1384-op units
-    alu_pipe_peak = SMS * 64 * peaks["sm_max_mhz"] * 1e6 / 1024 * SHA_OPS_PER_COMPRESSION / 1e12
+    alu_pipe_peak = sms * 64 * peaks["sm_max_mhz"] * 1e6 / 1024 * SHA_OPS_PER_COMPRESSION / 1e12
     achieved = (c_dig + c_chain) * SHA_OPS_PER_COMPRESSION / derive_s / 1e12
     table_s = float(np.mean(table_ms)) / 1e3
     # per key: 16 B key + one 32 B entry sector + 4 B new slot + 12 B of outputs (lookup slot, result,
@@ -530,7 +549,7 @@ def main():
                      "traffic": derive_traffic(args.workload),
                      "algorithmic_bytes": wl.batch.n_tokens * 4 + n_keys * 32,
                      "alu_pipe_peak": alu_pipe_peak,
-                     "peak_basis": f"{SMS} SMs x {LANES_PER_SM} int32 lanes x {peaks['sm_max_mhz']:.0f} MHz "
+                     "peak_basis": f"{sms} SMs (device query) x {LANES_PER_SM} int32 lanes x {peaks['sm_max_mhz']:.0f} MHz "
                                    f"(issue-rate ceiling); {SHA_OPS_PER_COMPRESSION} ops per compression, "
                                    f"{c_dig + c_chain} compressions per launch"},
         "probe_roofline": {"bound": "hbm", "kernel": "pk_lookup_store (probe + claim; finalize)",
@@ -547,9 +566,9 @@ def main():
                                    "ms_per_step": e2e_inplace_total / args.steps,
                                    "note": "all inputs read by the kernels from pinned host memory"}},
         # per step: chunk offsets, chunk+descriptor digests, chain; lookup-and-store (one kernel of
-        # request warps, or per key + per-request tail for few long requests); finalize
+        # request warps, or per key + per-request tail for few long requests); admit; finalize
         "critical_path": critical_path(wl, derive_s, peaks),
-        "gpu_launches": (3 + (1 if (R >= 1024 or N_cap <= 64 * R) else 2) + 1) * args.steps,
+        "gpu_launches": (3 + (1 if (R >= 1024 or N_cap <= 64 * R) else 2) + 2) * args.steps,
         "clocks": clk,
     }
     # Store-side omission test (comparison step, pk_compare_pages): 16,384 joined pages of 16 KiB against a
@@ -753,7 +772,7 @@ def main():
         "adapter_40MB_us": ad_us, "adapter_40MB_one_call_per_tensor_us": ad_single_us, "checkpoint_1GiB_us": ck_us,
         "checkpoint_GBps": ckpt_sizes[0] / (ck_us * 1e-6) / 1e9,
         "checkpoint_G_compressions_per_s": ck_comp / (ck_us * 1e-6) / 1e9,
-        "alu_pipe_peak_G_compressions_per_s": SMS * 64 * peaks["sm_max_mhz"] * 1e6 / 1024 / 1e9,
+        "alu_pipe_peak_G_compressions_per_s": sms * 64 * peaks["sm_max_mhz"] * 1e6 / 1024 / 1e9,
         "paper_host": "adapter 40 MB: 1.06 s cold, 0.060 s warm; 0.5B checkpoint content hash: 1.35 s"}
 
     # Two-level variant (request- and worker-level digests): the host cost of one request's digest under a

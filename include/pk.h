@@ -168,7 +168,9 @@ int pk_digest_descriptors(pk_ctx *ctx, const uint8_t *enc_dev, uint64_t enc_byte
                           const int64_t *enc_off_dev, uint32_t D, uint8_t *digests_dev,
                           int32_t *status_dev, pk_stream stream);
 
-/* Device.  Key derivation for R requests (steps c_i and k_i above).
+/* Device.  Key derivation for R requests: Key(x, c) = f(x, d) of Eq. 3
+ * (Sec. 5.2), f being the chained per-chunk digest of the header (steps c_i
+ * and k_i above), with keys only for full chunks (Sec. 4.4).
  *   tokens_dev   int32[n_tokens]
  *   tok_off_dev  int64[R+1], non-decreasing, tok_off[R] <= n_tokens;
  *                request r = tokens[tok_off[r], tok_off[r+1])
@@ -199,7 +201,10 @@ int pk_derive_keys_enc(pk_ctx *ctx, const int32_t *tokens_dev, uint64_t n_tokens
                        uint32_t D, uint8_t *digests_dev, int64_t *key_off_dev, uint8_t *keys_dev,
                        uint64_t key_capacity, int32_t *status_dev, pk_stream stream);
 
-/* Device.  Probe the table for every key of a pk_derive_keys result.
+/* Device.  The lookup of Sec. 2.1 (on a local miss the connector queries
+ * the shared store, and a hit skips that prefill), keyed by the 128-bit
+ * prefix of each k_i (Sec. 5.3: the digest is kept at 128 bits).  Probe the
+ * table for every key of a pk_derive_keys result.
  *   slots_dev       OUT uint32[key_capacity]: slot of key i, or PK_NO_SLOT
  *   hit_chunks_dev  OUT int32[R]: h_r = the largest j such that keys 0..j-1 of
  *                   request r are all present (the first miss ends the prefix);
@@ -210,7 +215,9 @@ int pk_lookup(pk_ctx *ctx, const uint8_t *keys_dev, const int64_t *key_off_dev, 
               uint64_t key_capacity, int32_t *hit_chunks_dev, uint32_t *slots_dev,
               int32_t *status_dev, pk_stream stream);
 
-/* Device.  Insert-if-absent of (prefix of keys_dev[e], slots_dev[e]), with
+/* Device.  The store of Sec. 2.1 (on a miss the connector computes the
+ * chunk's state and writes it to the shared store under the same key), over
+ * 128-bit key prefixes (Sec. 5.3).  Insert-if-absent of (prefix of keys_dev[e], slots_dev[e]), with
  * the outcome of processing the entries one by one in index order: an absent
  * key is inserted with its own slot (PK_STORE_INSERTED); a key already in the
  * table, or inserted by a lower index of the same call, keeps the existing
@@ -225,10 +232,13 @@ int pk_lookup(pk_ctx *ctx, const uint8_t *keys_dev, const int64_t *key_off_dev, 
  * slot_out_dev: uint32[n] (required: also holds intermediate positions).
  * Per-entry errors: PK_ERR_RESERVED_KEY, PK_ERR_ARG (slot == PK_NO_SLOT),
  * PK_ERR_TABLE_FULL, PK_ERR_PROBE_LIMIT; the first one also goes to
- * *status_dev.  A new key is refused once the table holds capacity - 1
- * entries.  Near that threshold, which of a call's new keys are refused is
- * unspecified, and insertions racing at it may take the last empty entries;
- * probes for absent keys then end at max_probe with PK_ERR_PROBE_LIMIT. */
+ * *status_dev.  Capacity: the table never holds more than capacity - 1
+ * entries (one always stays empty, so every probe ends), and refusals follow
+ * the index order too: with `room` = capacity - 1 - entries at the start of
+ * the call, the first `room` distinct new keys (ranked by their lowest
+ * index) are inserted and every entry of a later new key gets
+ * PK_ERR_TABLE_FULL.  A call that may not fit (entries + n >= capacity) adds
+ * a pass over its new keys, in index order when they do not all fit. */
 int pk_store(pk_ctx *ctx, const uint8_t *keys_dev, const uint32_t *slots_dev, uint64_t n,
              const int64_t *key_off_dev, const int32_t *hit_chunks_dev, uint32_t R,
              int32_t *result_dev, uint32_t *slot_out_dev, int32_t *status_dev, pk_stream stream);
@@ -417,8 +427,9 @@ int pk_table_load(pk_ctx *ctx, const void *src, size_t src_bytes, pk_stream stre
  * use (cudaMemset, or a table created by pk_init).  Arguments, results and
  * per-entry errors are those of pk_store, list or range mode.
  * No memory is allocated: the call's scratch (the table's entry count, the
- * latest call number in the table, and one 4-byte claim position per entry)
- * is a fixed file-scope device array of 16 + 4 * PK_NOALLOC_MAX_ENTRIES bytes
+ * latest call number in the table, the counts of the call's deferred and
+ * admitted keys, and one 4-byte claim position per entry) is a fixed
+ * file-scope device array of 32 + 4 * PK_NOALLOC_MAX_ENTRIES bytes
  * (about 1 MiB), held by every GPU that loads the library until the process
  * exits.  n > PK_NOALLOC_MAX_ENTRIES returns PK_ERR_TOO_LARGE before
  * anything is enqueued.  Each call first scans the whole table (count and

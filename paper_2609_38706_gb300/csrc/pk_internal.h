@@ -27,15 +27,17 @@ struct pk_ctx {
     uint32_t max_probe;
     uint64_t capacity;
     pk_entry *table;
-    unsigned long long *counter_dev;  // [0] entries in the table; [1] requests handed out by a lookup-and-store
+    unsigned long long *counter_dev;  // [0] entries in the table; [1] requests handed out by a lookup-and-store;
+                                      // [2] entries deferred in a store call; [3] keys its admit kernel claimed
     unsigned long long epoch;         // last store call number
     unsigned long long *stamps;       // budget mode: last-use stamp per entry (pk_attach_stamps), else NULL
     uint32_t pad_kw[64];              // K_t + W_t of a chunk's final (padding-only) block, C % 16 == 0
     uint32_t sm_count;                // SMs of the context's device (0 if unknown): picks the round form
 };
 
-// internal per-entry state between the two store kernels
-#define PK_STORE_PENDING 0x40000000
+// internal per-entry states between the store kernels (never returned)
+#define PK_STORE_PENDING 0x40000000   /* claimed or bid: the finalize kernel decides */
+#define PK_STORE_DEFERRED 0x40000001  /* absent, left to the admit kernel */
 
 // Launchers (pk_derive.cu, pk_table.cu).  Each returns the launch error.
 cudaError_t pk_launch_digest_descriptors(const uint8_t *enc, uint64_t enc_bytes, const int64_t *enc_off,

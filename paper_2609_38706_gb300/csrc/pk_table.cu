@@ -352,20 +352,44 @@ k_first_miss(const int64_t *key_off, uint32_t R, uint64_t key_capacity,
 }
 
 // ---------------------------------------------------------------------------
-// Store, kernel 1 of 2: find or claim each key's entry.
-//   pre-existing key (epoch of an earlier call): PRESENT with its slot, final
-//   key absent: CAS the key into the first empty entry
+// Store (Sec. 2.1: a miss computes and writes new state), with the outcome of
+// processing the entries one at a time in index order and at most
+// capacity - 1 entries ever stored.
+//
+// Claim kernel, for each entry:
+//   key inserted by an earlier call (epoch set, not this call's): PRESENT
+//   with its slot, final
 //   key claimed in this call (by anyone): bid (~index, slot) on the entry's
-//   slot/owner word and leave PENDING with the entry position in slot_out
-//   for kernel 2.
-// Capacity: when the table holds few enough entries that this call cannot
-// fill it (count + n < capacity), claims are counted once per block at the
-// end.  Otherwise a new key is refused (TABLE_FULL) once the count reaches
-// capacity - 1 and every claim is counted as it happens; claims racing at
-// that threshold can still take the last empty entries, after which probes
-// for absent keys end at max_probe (PK_ERR_PROBE_LIMIT).
+//   slot/owner word and leave PENDING with the entry position
+//   key absent: in claim mode, CAS the key into the first empty entry (then
+//   bid, PENDING); in defer mode, leave the entry DEFERRED for the admit
+//   kernel and write nothing
+// A warp takes claim mode when the entry count it reads plus the call's
+// entries stays below capacity: the whole call fits, so no key is refused.
+// (A warp that reads the count after other blocks added their claims may
+// take defer mode; its deferred keys then all fit as well.)
+// Admit kernel: nothing to do unless entries were deferred.  If the deferred
+// entries fit in the room left (capacity - 1 - count), all are claimed in
+// parallel; otherwise one CTA walks the deferred entries in index order,
+// each round letting at most `room` of them claim (so at most `room` new
+// keys), until the room is gone; the rest are bids on keys this call already
+// claimed, or TABLE_FULL.  That is exactly the sequential rule: the first
+// `room` distinct new keys (by lowest index) go in, later ones are refused.
+// Finalize kernel: each PENDING entry reads its key's slot/owner word, final
+// once every claim is in: the lowest claimant is INSERTED, the others
+// PRESENT with its slot.
+//
+// Context counter words: [0] entries in the table, [1] requests handed out
+// by a work-taking lookup-and-store, [2] entries deferred in this call,
+// [3] keys claimed by the admit kernel in this call (added to [0] and
+// cleared with [2] by the finalize kernel).
 // ---------------------------------------------------------------------------
 enum Examine { kAdvance, kDone, kClaimedHere };
+enum ClaimMode : uint32_t {
+    kModeClaim = 0,   // an absent key is claimed
+    kModeDefer = 1,   // an absent key is left DEFERRED (table not written)
+    kModeRefuse = 2,  // an absent key is refused (TABLE_FULL)
+};
 
 // Bid of entry index e (me = ~e) with its slot for a key new in this call:
 // the entry's slot/owner word ends at the maximum bid, that of the lowest
@@ -384,10 +408,8 @@ __device__ __forceinline__ void bid(pk_entry *ent, uint32_t me, uint32_t my_slot
 // the start of the call, or is inserted by it with a valid slot.
 template <bool kFused>
 __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cur, const uint4 &key, uint32_t me,
-                                           uint32_t my_slot, unsigned long long epoch, bool fast,
-                                           unsigned long long *counter, uint64_t capacity, bool may_claim,
-                                           unsigned long long *stamps, int32_t &res, uint32_t &out,
-                                           uint32_t &lslot) {
+                                           uint32_t my_slot, unsigned long long epoch, uint32_t mode, bool may_claim,
+                                           unsigned long long *stamps, int32_t &res, uint32_t &out, uint32_t &lslot) {
     uint4 *kp = reinterpret_cast<uint4 *>(ent->k);
     const unsigned long long my_stamp = (epoch << 32) | (unsigned long long)(uint32_t)~me;
     lslot = PK_NO_SLOT;
@@ -426,11 +448,9 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
             out = PK_NO_SLOT;
             return kDone;
         }
-        // Room check: refuse a new key once the table holds capacity - 1
-        // entries.  Only successful claims are counted (below), so racing
-        // duplicates of one key never touch the counter.
-        if (!fast && ld_volatile_u64(counter) + 1ull >= capacity) {
-            res = PK_ERR_TABLE_FULL;
+        if (mode != kModeClaim) {  // absent: left to the admit kernel, or refused
+            res = mode == kModeDefer ? PK_STORE_DEFERRED : PK_ERR_TABLE_FULL;
+            out = PK_NO_SLOT;
             return kDone;
         }
         const uint4 old = atomicCAS(kp, make_uint4(0, 0, 0, 0), key);
@@ -440,9 +460,7 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
             if (stamps) atomicMax(stamps + pos, my_stamp);
             res = PK_STORE_PENDING;
             out = (uint32_t)pos;
-            if (fast) return kClaimedHere;  // counted once per block at the end
-            atomicAdd(counter, 1ull);
-            return kDone;
+            return kClaimedHere;  // counted once per block at the end
         }
         cur = old;  // examine the winner's key
     }
@@ -461,17 +479,23 @@ struct ClaimCtx {
     pk_entry *table;
     uint64_t mask;
     uint32_t max_probe;
-    uint64_t capacity;
-    unsigned long long *counter;
     unsigned long long epoch;
-    bool fast;
+    uint32_t mode;               // ClaimMode: what happens to an absent key
     unsigned long long *stamps;  // budget mode: last-use stamp per entry, else NULL
 };
 
+// Mode of a claim kernel's warp: claim when the entry count plus the call's
+// entries stays below capacity (the whole call fits), else defer.
+__device__ __forceinline__ uint32_t claim_mode(const unsigned long long *counter, uint64_t n, uint64_t capacity) {
+    unsigned long long cnt = 0;
+    if ((threadIdx.x & 31) == 0) cnt = ld_volatile_u64(counter);
+    return __shfl_sync(kFull, cnt, 0) + n < capacity ? kModeClaim : kModeDefer;
+}
+
 // Insert-if-absent: one round over the undecided keys P of the warp.
 // Returns true in the lanes whose key was decided in this round, with its
-// result code and output; `claims` counts the fast-mode claims this lane
-// made as decider (for any key of the warp).
+// result code and output; `claims` counts the claims this lane made as
+// decider (for any key of the warp).
 // kFused: also `lslot`, the key's slot if it was in the table when the call
 // started (else PK_NO_SLOT), and keys with !may_claim are looked up only.
 template <bool kFused>
@@ -521,8 +545,8 @@ __device__ __forceinline__ bool claim_round(const ClaimCtx &c, uint32_t P, Probe
     uint32_t dprobed = 0;
     if (decider) {
         const uint64_t epos = wb + (uint32_t)cand;
-        const Examine x = examine<kFused>(c.table + epos, epos, cv, k, ~(uint32_t)we, wslot, c.epoch, c.fast,
-                                          c.counter, c.capacity, wmay, c.stamps, dres, dout, dls);
+        const Examine x = examine<kFused>(c.table + epos, epos, cv, k, ~(uint32_t)we, wslot, c.epoch, c.mode, wmay,
+                                          c.stamps, dres, dout, dls);
         if (x == kClaimedHere) ++claims;
         if (x == kAdvance) {  // lost the entry to a different key: continue after it
             dadv = true;
@@ -611,14 +635,18 @@ __device__ __forceinline__ bool in_store_range(const int64_t *key_off, const int
     return in_range;
 }
 
-// Adds the warp's fast-mode claims to the block total, then the block total
-// to the entry counter (same-address atomics serialise in L2).
-__device__ __forceinline__ void count_claims(unsigned long long *block_claims, uint32_t claims,
+// Adds the warp's claims and deferred entries to the block totals, then the
+// block totals to counter[0] (entries) and counter[2] (deferred): one atomic
+// per block and word (same-address atomics serialise in L2).
+__device__ __forceinline__ void count_claims(unsigned long long *block_sums, uint32_t claims, uint32_t deferred,
                                              unsigned long long *counter) {
     const uint32_t w = __reduce_add_sync(kFull, claims);
-    if ((threadIdx.x & 31) == 0 && w) atomicAdd_block(block_claims, (unsigned long long)w);
+    const uint32_t d = __reduce_add_sync(kFull, deferred);
+    if ((threadIdx.x & 31) == 0 && w) atomicAdd_block(block_sums, (unsigned long long)w);
+    if ((threadIdx.x & 31) == 0 && d) atomicAdd_block(block_sums + 1, (unsigned long long)d);
     __syncthreads();
-    if (threadIdx.x == 0 && *block_claims) atomicAdd(counter, *block_claims);
+    if (threadIdx.x == 0 && block_sums[0]) atomicAdd(counter, block_sums[0]);
+    if (threadIdx.x == 0 && block_sums[1]) atomicAdd(counter + 2, block_sums[1]);
 }
 
 // List mode, or range mode for few long requests: one warp per 32
@@ -629,18 +657,14 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
               const uint32_t *slots, uint64_t n, const int64_t *key_off,
               const int32_t *hit, uint32_t R, int32_t *result,
               uint32_t *slot_out, int32_t *status) {
-    __shared__ unsigned long long block_claims;
-    if (threadIdx.x == 0) block_claims = 0;
+    __shared__ unsigned long long block_sums[2];
+    if (threadIdx.x < 2) block_sums[threadIdx.x] = 0;
     __syncthreads();
     pk::pdl_wait(table, counter, keys, slots, key_off, hit, result, slot_out, status);
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const uint32_t lane = threadIdx.x & 31;
     bool active = e < n;
     if (key_off) active = in_store_range(key_off, hit, R, n, e) && active;
-    unsigned long long cnt = 0;
-    if (lane == 0) cnt = ld_volatile_u64(counter);
-    const bool fast = __shfl_sync(kFull, cnt, 0) + n < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast, stamps};
+    const ClaimCtx c{table, mask, max_probe, epoch, claim_mode(counter, n, capacity), stamps};
     int32_t res = PK_STORE_SKIPPED;
     uint32_t out = PK_NO_SLOT;
     ProbeKey s;
@@ -658,7 +682,7 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
         if (res < 0) set_status(status, res);
     }
     pk::pdl_launch_dependents();
-    count_claims(&block_claims, claims, counter);
+    count_claims(block_sums, claims, e < n && res == PK_STORE_DEFERRED, counter);
 }
 
 // Range mode for many short requests: one warp per request, no search.
@@ -670,8 +694,8 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
                   const uint32_t *slots, uint64_t n, const int64_t *key_off,
                   const int32_t *hit, uint32_t R, int32_t *result,
                   uint32_t *slot_out, int32_t *status) {
-    __shared__ unsigned long long block_claims;
-    if (threadIdx.x == 0) block_claims = 0;
+    __shared__ unsigned long long block_sums[2];
+    if (threadIdx.x < 2) block_sums[threadIdx.x] = 0;
     __syncthreads();
     pk::pdl_wait(table, counter, keys, slots, key_off, hit, result, slot_out, status);
     const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -684,11 +708,8 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
         const int64_t h0 = __ldcg(hit + r);
         first = a + (h0 > 0 ? h0 : 0);
     }
-    unsigned long long cnt = 0;
-    if (lane == 0) cnt = ld_volatile_u64(counter);
-    const bool fast = __shfl_sync(kFull, cnt, 0) + n < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast, stamps};
-    uint32_t claims = 0;
+    const ClaimCtx c{table, mask, max_probe, epoch, claim_mode(counter, n, capacity), stamps};
+    uint32_t claims = 0, deferred = 0;
     for (int64_t x = a + lane; x < first && x < b; x += 32) {  // below h_r: not stored
         result[x] = PK_STORE_SKIPPED;
         slot_out[x] = PK_NO_SLOT;
@@ -742,10 +763,11 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
             result[s.e] = res;
             slot_out[s.e] = out;
             if (res < 0) set_status(status, res);
+            deferred += res == PK_STORE_DEFERRED;
         }
     }
     pk::pdl_launch_dependents();
-    count_claims(&block_claims, claims, counter);
+    count_claims(block_sums, claims, deferred, counter);
 }
 
 // ---------------------------------------------------------------------------
@@ -767,7 +789,7 @@ __device__ __forceinline__ void lookup_store_request(const ClaimCtx &c, uint64_t
                                                      const uint32_t *new_slots, const int64_t *key_off, uint32_t R,
                                                      uint64_t key_capacity, uint32_t *slots, int32_t *hit,
                                                      int32_t *result, uint32_t *slot_out, int32_t *status,
-                                                     uint32_t &claims, bool release) {
+                                                     uint32_t &claims, uint32_t &deferred, bool release) {
     const uint64_t mask = c.mask;
     const uint32_t lane = threadIdx.x & 31;
     int64_t a = 0, b = 0;
@@ -826,6 +848,7 @@ __device__ __forceinline__ void lookup_store_request(const ClaimCtx &c, uint64_t
             slots[e] = lslot;
             result[e] = res;
             slot_out[e] = out;
+            deferred += res == PK_STORE_DEFERRED;
             if (lslot == PK_NO_SLOT) {
                 first_miss = min(first_miss, (uint32_t)(e - a));
                 if (res < 0) set_status(status, res);
@@ -865,27 +888,23 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
                    const uint32_t *new_slots, const int64_t *key_off, uint32_t R,
                    uint64_t key_capacity, uint32_t *slots, int32_t *hit,
                    int32_t *result, uint32_t *slot_out, int32_t *status, unsigned long long *tickets) {
-    __shared__ unsigned long long block_claims;
-    if (threadIdx.x == 0) block_claims = 0;
+    __shared__ unsigned long long block_sums[2];
+    if (threadIdx.x < 2) block_sums[threadIdx.x] = 0;
     __syncthreads();
     pk::pdl_wait(table, counter, keys, new_slots, key_off, slots, hit, result, slot_out, status, tickets);
-    const uint32_t lane = threadIdx.x & 31;
-    unsigned long long cnt = 0;
-    if (lane == 0) cnt = ld_volatile_u64(counter);
-    const bool fast = __shfl_sync(kFull, cnt, 0) + key_capacity < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast, stamps};
-    uint32_t claims = 0;
+    const ClaimCtx c{table, mask, max_probe, epoch, claim_mode(counter, key_capacity, capacity), stamps};
+    uint32_t claims = 0, deferred = 0;
     if (kTake) {
         for (uint64_t r = take_request(tickets); r < R; r = take_request(tickets))
             lookup_store_request(c, r, keys, new_slots, key_off, R, key_capacity, slots, hit, result, slot_out,
-                                 status, claims, false);
+                                 status, claims, deferred, false);
         pk::pdl_launch_dependents();
     } else {
         const uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
         lookup_store_request(c, r, keys, new_slots, key_off, R, key_capacity, slots, hit, result, slot_out, status,
-                             claims, true);
+                             claims, deferred, true);
     }
-    count_claims(&block_claims, claims, counter);
+    count_claims(block_sums, claims, deferred, counter);
 }
 
 // Few long requests: one warp per 32 consecutive keys; k_lookup_store_tail
@@ -895,18 +914,14 @@ k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capa
                unsigned long long epoch, unsigned long long *stamps, const uint8_t *keys, const uint32_t *new_slots,
                const int64_t *key_off, uint32_t R, uint64_t key_capacity, uint32_t *slots,
                int32_t *result, uint32_t *slot_out, int32_t *status) {
-    __shared__ unsigned long long block_claims;
-    if (threadIdx.x == 0) block_claims = 0;
+    __shared__ unsigned long long block_sums[2];
+    if (threadIdx.x < 2) block_sums[threadIdx.x] = 0;
     __syncthreads();
     pk::pdl_wait(table, counter, keys, new_slots, key_off, slots, result, slot_out, status);
     const int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const uint32_t lane = threadIdx.x & 31;
     const int64_t total = R == 0 ? 0 : __ldcg(key_off + R);
     const int64_t end = total < (int64_t)key_capacity ? total : (int64_t)key_capacity;
-    unsigned long long cnt = 0;
-    if (lane == 0) cnt = ld_volatile_u64(counter);
-    const bool fast = __shfl_sync(kFull, cnt, 0) + key_capacity < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, counter, epoch, fast, stamps};
+    const ClaimCtx c{table, mask, max_probe, epoch, claim_mode(counter, key_capacity, capacity), stamps};
     int32_t res = PK_STORE_SKIPPED;
     uint32_t out = PK_NO_SLOT, lslot = PK_NO_SLOT;
     ProbeKey s;
@@ -928,7 +943,7 @@ k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capa
         if (lslot == PK_NO_SLOT && res < 0) set_status(status, res);
     }
     pk::pdl_launch_dependents();
-    count_claims(&block_claims, claims, counter);
+    count_claims(block_sums, claims, e < end && res == PK_STORE_DEFERRED, counter);
 }
 
 // One warp per request: h_r = the first miss (slot PK_NO_SLOT), entries below
@@ -965,16 +980,140 @@ k_lookup_store_tail(const int64_t *key_off, uint32_t R, uint64_t key_capacity,
     if (arg) set_status(status, PK_ERR_ARG);
 }
 
-// Store, kernel 2 of 2: each PENDING entry reads its key's slot/owner word,
+// Result of a deferred entry decided by the admit kernel.  pos_out: where a
+// PENDING entry's table position goes (slot_out for a context; the
+// allocation-free store keeps positions apart and writes PK_NO_SLOT to
+// slot_out).
+__device__ __forceinline__ void admit_write(uint64_t e, int32_t res, uint32_t out, int32_t *result,
+                                            uint32_t *slot_out, uint32_t *pos_out, int32_t *status) {
+    result[e] = res;
+    if (res == PK_STORE_PENDING && pos_out != slot_out) {
+        pos_out[e] = out;
+        slot_out[e] = PK_NO_SLOT;
+    } else {
+        slot_out[e] = out;
+    }
+    if (res < 0) set_status(status, res);
+}
+
+// Store, admit kernel (see the store comment above).  The call's entries are
+// [0, n), or [0, min(n, key_off[R])) in range and lookup-and-store mode;
+// counter[0] is the entry count after the claim kernel, counter[2] the
+// number of DEFERRED entries; keys claimed here are added to counter[3].
+// Within the call the entry count can only reach capacity - 1: the claim
+// kernel claims only when the whole call fits, and here at most `room` keys
+// are claimed.
+__device__ __forceinline__ void store_admit(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
+                                            unsigned long long *counter, unsigned long long epoch,
+                                            unsigned long long *stamps, const uint8_t *keys, const uint32_t *slots,
+                                            uint64_t n, const int64_t *key_off, uint32_t R, int32_t *result,
+                                            uint32_t *slot_out, uint32_t *pos_out, int32_t *status) {
+    __shared__ uint32_t s_warp[8];
+    __shared__ unsigned long long s_claims;
+    const unsigned long long deferred = __ldcg(counter + 2);
+    if (deferred == 0) return;  // every key was decided by the claim kernel
+    const unsigned long long count = __ldcg(counter);
+    const unsigned long long room = count + 1 < capacity ? capacity - 1 - count : 0ull;
+    uint64_t end = n;
+    if (key_off) {
+        const int64_t t = R ? __ldcg(key_off + R) : 0;
+        if (t < (int64_t)end) end = t > 0 ? (uint64_t)t : 0;
+    }
+    const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (deferred <= room) {
+        // At most `deferred` distinct keys: all fit.  Claimed in parallel.
+        const ClaimCtx c{table, mask, max_probe, epoch, kModeClaim, stamps};
+        uint32_t claims = 0;
+        if (threadIdx.x == 0) s_claims = 0;
+        __syncthreads();
+        for (uint64_t base = (uint64_t)blockIdx.x * blockDim.x + 32 * warp; base < end;
+             base += (uint64_t)gridDim.x * blockDim.x) {  // uniform per warp
+            const uint64_t e = base + lane;
+            ProbeKey s;
+            s.pending = false;
+            if (e < end && __ldcg(result + e) == PK_STORE_DEFERRED)
+                probe_start(s, ld_cg_v4(keys + 32 * e), e, mask, __ldcg(slots + e));
+            const bool mine = s.pending;
+            int32_t res;
+            uint32_t out, lslot;
+            warp_claim<false>(c, s, res, out, lslot, claims);
+            if (mine) admit_write(e, res, out, result, slot_out, pos_out, status);
+        }
+        const uint32_t wc = __reduce_add_sync(kFull, claims);
+        if (lane == 0 && wc) atomicAdd_block(&s_claims, (unsigned long long)wc);
+        __syncthreads();
+        if (threadIdx.x == 0 && s_claims) atomicAdd(counter + 3, s_claims);
+        return;
+    }
+    // More deferred entries than room: one CTA walks them in index order, 256
+    // at a time.  Each round the first `left` undecided entries of the tile
+    // (at most `left` distinct keys) claim or bid; once the room is gone the
+    // rest only bid on keys this call claimed, or are refused.  Every round
+    // decides at least one entry.
+    if (blockIdx.x != 0) return;
+    unsigned long long left = room, admitted = 0;
+    for (uint64_t base = 0; base < end; base += blockDim.x) {
+        const uint64_t e = base + threadIdx.x;
+        bool pend = e < end && __ldcg(result + e) == PK_STORE_DEFERRED;
+        const uint4 key = pend ? ld_cg_v4(keys + 32 * e) : make_uint4(0, 0, 0, 0);
+        const uint32_t sl = pend ? __ldcg(slots + e) : 0u;
+        for (;;) {
+            const uint32_t ball = __ballot_sync(kFull, pend);
+            if (lane == 0) s_warp[warp] = __popc(ball);
+            if (threadIdx.x == 0) s_claims = 0;
+            if (__syncthreads_count(pend) == 0) break;  // the tile is decided (uniform)
+            uint32_t rank = __popc(ball & lanemask_lt());
+            for (uint32_t w = 0; w < warp; ++w) rank += s_warp[w];
+            const bool act = pend && (left == 0 || rank < left);
+            const ClaimCtx c{table, mask, max_probe, epoch, left == 0 ? kModeRefuse : kModeClaim, stamps};
+            ProbeKey s;
+            s.pending = false;
+            if (act) probe_start(s, key, e, mask, sl);
+            uint32_t claims = 0;
+            int32_t res;
+            uint32_t out, lslot;
+            warp_claim<false>(c, s, res, out, lslot, claims);
+            if (act) {
+                admit_write(e, res, out, result, slot_out, pos_out, status);
+                pend = false;
+            }
+            const uint32_t wc = __reduce_add_sync(kFull, claims);
+            if (lane == 0 && wc) atomicAdd_block(&s_claims, (unsigned long long)wc);
+            __syncthreads();
+            left -= s_claims;  // <= left: at most `left` entries claimed
+            admitted += s_claims;
+            __syncthreads();  // s_warp and s_claims are rewritten next round
+        }
+    }
+    if (threadIdx.x == 0 && admitted) atomicAdd(counter + 3, admitted);
+}
+
+__global__ void __launch_bounds__(256)
+k_store_admit(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity, unsigned long long *counter,
+              unsigned long long epoch, unsigned long long *stamps, const uint8_t *keys, const uint32_t *slots,
+              uint64_t n, const int64_t *key_off, uint32_t R, int32_t *result, uint32_t *slot_out, int32_t *status) {
+    pk::pdl_launch_dependents();
+    pk::pdl_wait(table, counter, stamps, keys, slots, key_off, result, slot_out, status);
+    store_admit(table, mask, max_probe, capacity, counter, epoch, stamps, keys, slots, n, key_off, R, result,
+                slot_out, slot_out, status);
+}
+
+// Store, last kernel: each PENDING entry reads its key's slot/owner word,
 // final once every claim is in: the lowest claimant is INSERTED, the others
 // PRESENT with its slot.  In range mode, entries past key_off[R] (not keys
-// of this batch) are skipped.
+// of this batch) are skipped.  The admit kernel's claims are added to the
+// entry count, and the call's counter words [2] and [3] cleared.
 __global__ void __launch_bounds__(256)
 k_store_finalize(const pk_entry *table, uint64_t n, const int64_t *key_off, uint32_t R,
-                 int32_t *result, uint32_t *slot_out) {
+                 int32_t *result, uint32_t *slot_out, unsigned long long *counter) {
     pk::pdl_launch_dependents();
-    pk::pdl_wait(table, key_off, result, slot_out);
+    pk::pdl_wait(table, key_off, result, slot_out, counter);
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e == 0 && __ldcg(counter + 2)) {
+        counter[0] += __ldcg(counter + 3);
+        counter[2] = 0;
+        counter[3] = 0;
+    }
     if (e >= n) return;
     if (key_off && (int64_t)e >= (R > 0 ? __ldcg(key_off + R) : 0)) {
         result[e] = PK_STORE_SKIPPED;
@@ -1032,8 +1171,11 @@ __global__ void k_mark_loaded(pk_entry *table, uint64_t capacity) {
 // positions live in this one file-scope array, shared by every call.
 // ---------------------------------------------------------------------------
 struct NoallocScratch {
-    unsigned long long count;      // entries in the table (set by the scan, then claims)
-    unsigned long long epoch_max;  // largest call number found in the table
+    // [0] entries in the table (set by the scan, then claims), [1] largest
+    // call number found in the table, [2] entries deferred in this call,
+    // [3] keys its admit kernel claimed: [0], [2] and [3] are the words a
+    // context's counter holds at the same indices
+    unsigned long long word[4];
     uint32_t pos[PK_NOALLOC_MAX_ENTRIES];  // table position of each PENDING entry
 };
 static __device__ __align__(256) NoallocScratch g_noalloc_scratch;
@@ -1058,8 +1200,8 @@ k_noalloc_scan(const pk_entry *table, uint64_t capacity, NoallocScratch *sc) {
     atomicMax_block(&blk_epoch, ep);
     __syncthreads();
     if (threadIdx.x == 0) {
-        if (blk_count) atomicAdd(&sc->count, blk_count);
-        atomicMax(&sc->epoch_max, blk_epoch);
+        if (blk_count) atomicAdd(&sc->word[0], blk_count);
+        atomicMax(&sc->word[1], blk_epoch);
     }
 }
 
@@ -1071,18 +1213,14 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
                 const uint8_t *keys, const uint32_t *slots, uint64_t n,
                 const int64_t *key_off, const int32_t *hit, uint32_t R,
                 int32_t *result, uint32_t *slot_out, int32_t *status) {
-    __shared__ unsigned long long block_claims;
-    if (threadIdx.x == 0) block_claims = 0;
+    __shared__ unsigned long long block_sums[2];
+    if (threadIdx.x < 2) block_sums[threadIdx.x] = 0;
     __syncthreads();
-    const unsigned long long epoch = ld_volatile_u64(&sc->epoch_max) + 1ull;
+    const unsigned long long epoch = ld_volatile_u64(&sc->word[1]) + 1ull;
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const uint32_t lane = threadIdx.x & 31;
     bool active = e < n;
     if (key_off) active = in_store_range(key_off, hit, R, n, e) && active;
-    unsigned long long cnt = 0;
-    if (lane == 0) cnt = ld_volatile_u64(&sc->count);
-    const bool fast = __shfl_sync(kFull, cnt, 0) + n < capacity;
-    const ClaimCtx c{table, mask, max_probe, capacity, &sc->count, epoch, fast, nullptr};
+    const ClaimCtx c{table, mask, max_probe, epoch, claim_mode(sc->word, n, capacity), nullptr};
     int32_t res = PK_STORE_SKIPPED;
     uint32_t out = PK_NO_SLOT;
     ProbeKey s;
@@ -1104,7 +1242,18 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
         }
         if (res < 0) set_status(status, res);
     }
-    count_claims(&block_claims, claims, &sc->count);
+    count_claims(block_sums, claims, e < n && res == PK_STORE_DEFERRED, sc->word);
+}
+
+// The admit kernel of the allocation-free store: the call number comes
+// from scratch, and PENDING positions go there.
+__global__ void __launch_bounds__(256)
+k_noalloc_admit(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity, NoallocScratch *sc,
+                const uint8_t *keys, const uint32_t *slots, uint64_t n, const int64_t *key_off, uint32_t R,
+                int32_t *result, uint32_t *slot_out, int32_t *status) {
+    const unsigned long long epoch = ld_volatile_u64(&sc->word[1]) + 1ull;
+    store_admit(table, mask, max_probe, capacity, sc->word, epoch, nullptr, keys, slots, n, key_off, R, result,
+                slot_out, sc->pos, status);
 }
 
 __global__ void __launch_bounds__(256)
@@ -1118,6 +1267,14 @@ k_noalloc_finalize(const pk_entry *table, const NoallocScratch *sc, uint64_t n, 
 }
 
 unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1) / block); }
+
+// Grid of the admit kernel: grid-strided, at most two CTAs per SM (a launch
+// that usually finds nothing to do).
+unsigned admit_grid(uint64_t n, uint32_t sms) {
+    const unsigned g = grid_for(n, 256);
+    const unsigned cap = sms ? 2u * sms : g;
+    return g < cap ? g : (cap ? cap : 1u);
+}
 
 // Per-request kernels when the batch has many short requests; per-key kernels
 // when a few requests carry many keys each (a warp per request would then
@@ -1200,8 +1357,12 @@ cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const u
                       ctx->counter_dev, epoch, ctx->stamps, keys, slots, n, key_off, hit_chunks, R, result, slot_out, status);
     }
     if (e == cudaSuccess)
+        e = pk_launch(k_store_admit, admit_grid(n, ctx->sm_count), 256, s, ctx->table, mask, ctx->max_probe,
+                      ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, slots, n, key_off, R, result,
+                      slot_out, status);
+    if (e == cudaSuccess)
         e = pk_launch(k_store_finalize, grid_for(n, 256), 256, s, (const pk_entry *)ctx->table, n, key_off, R, result,
-                      slot_out);
+                      slot_out, ctx->counter_dev);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -1239,8 +1400,12 @@ cudaError_t pk_launch_lookup_store(const pk_ctx *ctx, unsigned long long epoch, 
                           (const uint32_t *)slots, hit_chunks, result, slot_out, status);
     }
     if (e == cudaSuccess && key_capacity)
+        e = pk_launch(k_store_admit, admit_grid(key_capacity, ctx->sm_count), 256, s, ctx->table, mask,
+                      ctx->max_probe, ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, new_slots,
+                      key_capacity, key_off, R, result, slot_out, status);
+    if (e == cudaSuccess && key_capacity)
         e = pk_launch(k_store_finalize, grid_for(key_capacity, 256), 256, s, (const pk_entry *)ctx->table,
-                      key_capacity, key_off, R, result, slot_out);
+                      key_capacity, key_off, R, result, slot_out, ctx->counter_dev);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -1286,15 +1451,18 @@ cudaError_t pk_launch_store_noalloc(pk_entry *table, uint32_t capacity_log2, uin
     if (!sc) return cudaErrorInvalidSymbol;
     if (n == 0) return cudaSuccess;
     const uint64_t capacity = 1ull << capacity_log2;
-    // count and epoch_max must start at zero; pos needs no clearing
-    e = cudaMemsetAsync(sc, 0, 2 * sizeof(unsigned long long), s);
+    // the four counter words must start at zero; pos needs no clearing
+    e = cudaMemsetAsync(sc, 0, sizeof sc->word, s);
     if (e != cudaSuccess) return e;
     const uint64_t scan_blocks = (capacity + 255) / 256;
     const uint32_t sms = device_sms(device);
     const uint64_t scan_cap = sms ? 8ull * sms : scan_blocks;  // grid-strided: any grid is correct
+    const uint32_t Rm = key_off ? R : 0;
     k_noalloc_scan<<<(unsigned)(scan_blocks < scan_cap ? scan_blocks : scan_cap), 256, 0, s>>>(table, capacity, sc);
     k_noalloc_claim<<<grid_for(n, 256), 256, 0, s>>>(table, capacity - 1, max_probe, capacity, sc, keys, slots, n,
-                                                      key_off, hit_chunks, key_off ? R : 0, result, slot_out, status);
+                                                      key_off, hit_chunks, Rm, result, slot_out, status);
+    k_noalloc_admit<<<admit_grid(n, sms), 256, 0, s>>>(table, capacity - 1, max_probe, capacity, sc, keys, slots, n,
+                                                        key_off, Rm, result, slot_out, status);
     k_noalloc_finalize<<<grid_for(n, 256), 256, 0, s>>>(table, sc, n, result, slot_out);
     return cudaGetLastError();
 }

@@ -59,3 +59,12 @@ def test_critical_path_of_the_multi_adapter_batch():
 def test_ops_per_compression():
     # 64 rounds x (6 rotations + 4 three-input logic + 4 adds) + 48 schedule words x (6 + 2 + 2) + 8 feed-forward
     assert bench.SHA_OPS_PER_COMPRESSION == 64 * 14 + 48 * 10 + 8 == 1384
+
+
+def test_auto_steps_give_a_timed_region_of_at_least_the_minimum():
+    import bench
+    for it in (0.2e-3, 0.9e-3, 1.4e-3, 7e-3):
+        k = bench.auto_steps(it)
+        assert k * it >= bench.MIN_TIMED_S or k == 4000
+        assert (k - 1) * it < bench.MIN_TIMED_S or k == 20
+    assert bench.auto_steps(10.0) == 20 and bench.auto_steps(1e-9) == 4000 and bench.auto_steps(0) == 20

@@ -14,7 +14,8 @@ pytestmark = pytest.mark.gpu
 
 REDUCED = ["tiny", "multi_adapter", "small_block", "long_context", "provenance_sweep_D1",
            "provenance_sweep_D4", "provenance_sweep_D16", "provenance_sweep_D64"]
-FULL = ["multi_adapter", "small_block", "long_context", "provenance_sweep_D4"]
+FULL = ["multi_adapter", "small_block", "long_context", "provenance_sweep_D1", "provenance_sweep_D4",
+        "provenance_sweep_D16", "provenance_sweep_D64"]
 
 
 @pytest.fixture(scope="module", autouse=True)
