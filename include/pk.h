@@ -397,6 +397,20 @@ int pk_key_strings(const uint8_t *keys_dev, uint64_t n, const char *prefix, uint
  *                     written); PK_ERR_TIMEOUT (table unspecified).  One
  *                     cooperative launch; within the budget it returns at
  *                     once. */
+/* Test hook of pk_evict's bounded grid barriers (no paper counterpart): the
+ * same launch as pk_evict(ctx, budget, budget, ...) with the barrier waits
+ * bounded at spin_limit polls of about 100-200 ns (> 0; at most the default
+ * of about a second) and CTA 0 withholding its arrival at the first barrier,
+ * so that every other CTA's wait runs out.  Needs stamps attached and more
+ * than `budget` entries in the table (else the kernel returns before the
+ * barrier) and a table of at least 2^10 entries (two CTAs or more).  The
+ * launch must end by itself with PK_ERR_TIMEOUT in *status_dev; the first
+ * barrier precedes every write to the table and the stamps, so both are
+ * unchanged, and the context stays usable.  Errors (host): PK_ERR_ARG,
+ * PK_ERR_CUDA. */
+int pk_evict_barrier_timeout_test(pk_ctx *ctx, uint64_t budget, void *scratch_dev, size_t scratch_bytes,
+                                  uint32_t spin_limit, int32_t *status_dev, pk_stream stream);
+
 size_t pk_stamps_bytes(uint32_t capacity_log2);
 int pk_attach_stamps(pk_ctx *ctx, uint64_t *stamps_dev, size_t stamps_bytes, pk_stream stream);
 size_t pk_evict_scratch_bytes(uint32_t capacity_log2);
@@ -428,8 +442,8 @@ int pk_table_load(pk_ctx *ctx, const void *src, size_t src_bytes, pk_stream stre
  * per-entry errors are those of pk_store, list or range mode.
  * No memory is allocated: the call's scratch (the table's entry count, the
  * latest call number in the table, the counts of the call's deferred and
- * admitted keys, and one 4-byte claim position per entry) is a fixed
- * file-scope device array of 32 + 4 * PK_NOALLOC_MAX_ENTRIES bytes
+ * claimed keys, and one 4-byte claim position per entry) is a fixed
+ * file-scope device array of 40 + 4 * PK_NOALLOC_MAX_ENTRIES bytes
  * (about 1 MiB), held by every GPU that loads the library until the process
  * exits.  n > PK_NOALLOC_MAX_ENTRIES returns PK_ERR_TOO_LARGE before
  * anything is enqueued.  Each call first scans the whole table (count and

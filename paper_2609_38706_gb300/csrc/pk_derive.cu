@@ -13,6 +13,8 @@
 // and overwritten in place by the chain, so derivation needs no scratch memory.
 #include <cuda_runtime.h>
 
+#include <mutex>
+
 #include "pk_device.cuh"
 #include "pk_internal.h"
 #include "pk_sha256.cuh"
@@ -313,24 +315,37 @@ k_chunk_digest(const int32_t *tokens, const int64_t *tok_off,
 // ---------------------------------------------------------------------------
 // Chain: k_i = SHA-256(k_{i-1} || d || c_i), serial in i for each request.
 //
-// Each CTA serves 32 requests (one per lane) with two warps on different SM
-// sub-partitions, so that one chain step costs about the rounds alone:
-//   warp 0 (rounds):   holds the state; runs the 64 rounds of block 1
-//                      (k_{i-1} || d) and of block 2 (c_i || padding)
-//   warp 1 (schedule): writes K_t + W_t for both blocks to shared memory:
-//                      block 2's schedule depends on c_i only and is made one
-//                      step ahead; block 1's depends on k_{i-1} and is made in
-//                      three 16-word slices as soon as k_{i-1} is published.
-// Named barriers (count 64 = both warps), producer arrives / consumer syncs:
-//   1, 2, 3  block-1 slices t = 16..31, 32..47, 48..63 of step i are ready
-//   4        block-2 schedule of step i is ready
-//   5        k_i is published (rounds warp -> schedule warp)
-// Per CTA both warps run the same number of steps (the lanes' maximum), so
+// Every 32 requests (one per lane, a "group") are served by a pair of warps:
+//   rounds warp:   holds the state; runs the 64 rounds of block 1
+//                  (k_{i-1} || d) and of block 2 (c_i || padding)
+//   schedule warp: writes K_t + W_t for both blocks to shared memory:
+//                  block 2's schedule depends on c_i only and is made one
+//                  step ahead; block 1's depends on k_{i-1} and is made as
+//                  soon as k_{i-1} is published.
+// Two layouts (kPairs):
+//   1  one pair per CTA (2 warps) for batches with at most one group per SM:
+//      the two warps run on different SM sub-partitions, so that one chain
+//      step costs about the rounds alone; block 1's schedule is published in
+//      three 16-word slices.  Named barriers (count 64, producer arrives,
+//      consumer syncs): 1, 2, 3 block-1 slices t = 16..31, 32..47, 48..63;
+//      4 block-2 schedule; 5 k_i published.
+//   4  four pairs per CTA (8 warps), pair p = rounds warp p and schedule warp
+//      p + 4, which share a sub-partition, one CTA per SM: with several
+//      groups per SM, 2-warp CTAs put two rounds warps on one sub-partition
+//      (51 instead of 30 cycles per round, measured) while schedule warps
+//      share another; paired on one sub-partition, the schedule fills the
+//      issue slots the rounds warp's dependency chain leaves idle.  Block 1's
+//      schedule is published in one piece.  Named barriers of pair p:
+//      1 + 3p block-1 schedule; 2 + 3p block-2 schedule; 3 + 3p k_i published.
+// Per pair both warps run the same number of steps (the lanes' maximum), so
 // every phase of every barrier gets exactly one arrive and one sync; the
-// schedule warp signals barrier 4 for step i only after it has passed barrier
-// 5 of step i-1, so it never arrives twice on a barrier the rounds warp has
-// not yet synced.  Lanes past their own request's last chunk keep computing
-// (masked) so that the warps stay aligned.
+// schedule warp signals the block-2 barrier for step i only after it has
+// passed the k barrier of step i-1 (so after the rounds warp has synced the
+// block-2 barrier of step i-1), and the block-1 barrier of step i only after
+// the k barrier of step i-1 (after the rounds warp's block-1 sync of step
+// i-1): it never arrives twice on a barrier the rounds warp has not yet
+// synced.  Lanes past their own request's last chunk keep computing (masked)
+// so that the warps stay aligned.
 // ---------------------------------------------------------------------------
 constexpr int kChainLanes = 32;
 
@@ -344,11 +359,14 @@ struct ChainSmem {
 };
 
 // 16 schedule words t = 16q .. 16q+15 of the ring w (in place), K_t + W_t -> out[t][lane]
-__device__ __forceinline__ void schedule16(uint32_t w[16], uint32_t (*out)[kChainLanes], int q, uint32_t lane) {
+// (F: round form of pk_sha256.cuh, `one` its run-time 1)
+template <int F>
+__device__ __forceinline__ void schedule16(uint32_t w[16], uint32_t (*out)[kChainLanes], int q, uint32_t lane,
+                                           uint32_t one) {
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
-        w[j] += pk::small_s1(w[(j + 14) & 15]) + w[(j + 9) & 15] + pk::small_s0(w[(j + 1) & 15]);
-        out[16 * q + j][lane] = pk::kSha256K[16 * q + j] + w[j];
+        pk::sched_word<F>(w, j, one);
+        out[16 * q + j][lane] = pk::add2<F>(pk::kSha256K[16 * q + j], w[j], one);
     }
 }
 
@@ -356,40 +374,68 @@ __device__ __forceinline__ void schedule16(uint32_t w[16], uint32_t (*out)[kChai
 // (the 16 words are read into registers before the first round: a lone warp
 // runs 64 rounds in 2018 instead of 2241 cycles when no round waits on its
 // shared-memory read)
-__device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint32_t (*kw)[kChainLanes], int q, uint32_t lane) {
+template <int F>
+__device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint32_t (*kw)[kChainLanes], int q, uint32_t lane,
+                                            uint32_t one) {
     uint32_t a = v[0], b = v[1], c = v[2], d = v[3], e = v[4], f = v[5], g = v[6], h = v[7];
     uint32_t x[16];
 #pragma unroll
     for (int j = 0; j < 16; ++j) x[j] = kw[16 * q + j][lane];
 #pragma unroll
-    for (int j = 0; j < 16; ++j) pk::round_kw(a, b, c, d, e, f, g, h, x[j]);
+    for (int j = 0; j < 16; ++j) pk::round_kw<F>(a, b, c, d, e, f, g, h, x[j], one);
     v[0] = a; v[1] = b; v[2] = c; v[3] = d; v[4] = e; v[5] = f; v[6] = g; v[7] = h;
 }
 
-// At most 64 registers (15 CTAs per SM, no spills): uncapped, the compiler took 81 and a small-block
-// step whose lookup-and-store launch overlaps the chain's tail ran 910 -> 955 us.
-__global__ void __launch_bounds__(2 * kChainLanes, 15)
+// At most 64 registers (no spills): uncapped, the compiler took 81 and a small-block step whose
+// lookup-and-store launch overlaps the chain's tail ran 910 -> 955 us.  `groups` = ceil(R / 32); with
+// kPairs = 4, CTA c serves groups [c * groups / gridDim.x, (c + 1) * groups / gridDim.x), at most four.
+// FS: the form (pk_sha256.cuh) of the schedule warp's additions, `one` its run-time 1.  The rounds warp
+// keeps the compiler's form: its dependency chain sets the step time, and a multiply-add's longer latency
+// there made the four-pair chain slower (small-block key derivation 674 -> 718 us with every addition on the
+// FMA pipe).  With four pairs each sub-partition runs a rounds and a schedule warp on one ALU pipe, so the
+// schedule warp's additions go to the FMA pipe.
+template <int kPairs, int FS>
+__global__ void __launch_bounds__(2 * kChainLanes * kPairs, kPairs == 1 ? 15 : 4)
 k_chain(const int64_t *key_off, const uint32_t *desc_idx,
-        const uint8_t *digests, uint32_t R, uint32_t D, uint8_t *keys) {
-    __shared__ __align__(16) ChainSmem sm;
+        const uint8_t *digests, uint32_t R, uint32_t D, uint8_t *keys, uint32_t groups, uint32_t one) {
+    extern __shared__ __align__(16) uint8_t chain_smem[];
     pk::pdl_wait(key_off, desc_idx, digests, keys);  // successor released at the last step (see k_chunk_digest)
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const uint32_t r = blockIdx.x * kChainLanes + lane;
+    const uint32_t pair = kPairs == 1 ? 0u : warp & (kPairs - 1);
+    const bool sched = kPairs == 1 ? warp == 1 : warp >= (uint32_t)kPairs;
+    ChainSmem &sm = reinterpret_cast<ChainSmem *>(chain_smem)[pair];
+    uint32_t group = blockIdx.x;
+    bool active = true;
+    if (kPairs > 1) {
+        const uint32_t g0 = (uint32_t)((uint64_t)blockIdx.x * groups / gridDim.x);
+        const uint32_t g1 = (uint32_t)((uint64_t)(blockIdx.x + 1) * groups / gridDim.x);
+        group = g0 + pair;
+        active = group < g1;
+    }
+    // named barriers of this pair (compile-time ids with one pair per CTA)
+    const int bar_s1 = kPairs == 1 ? 1 : 1 + 3 * (int)pair;  // block-1 schedule (first slice)
+    const int bar_b2 = kPairs == 1 ? 4 : 2 + 3 * (int)pair;  // block-2 schedule
+    const int bar_k = kPairs == 1 ? 5 : 3 + 3 * (int)pair;   // k_i published
+    const uint32_t r = group * kChainLanes + lane;
     int64_t a = 0, n = 0;
     uint32_t di = 0;
-    if (r < R) {
+    if (active && r < R) {
         a = key_off[r];
         n = key_off[r + 1] - a;
         di = desc_idx[r];
         if (n < 0 || di >= D) n = 0;
     }
-    int64_t nmax = n;  // identical in both warps: they cover the same 32 requests
+    int64_t nmax = n;  // identical in both warps of the pair: they cover the same 32 requests
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         const int64_t x = __shfl_xor_sync(0xffffffffu, nmax, o);
         nmax = x > nmax ? x : nmax;
     }
-    if (nmax == 0) return;  // uniform over the CTA
+    if (nmax == 0) {  // uniform over the pair
+        pk::pdl_launch_dependents();
+        if (kPairs > 1) __syncthreads();
+        return;
+    }
 
     uint32_t dw[8] = {0, 0, 0, 0, 0, 0, 0, 0};
     if (n > 0) {
@@ -401,7 +447,7 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
     }
     uint4 *kq = reinterpret_cast<uint4 *>(keys + 32ull * a);
 
-    if (warp == 1) {  // ---------------- schedule warp ----------------
+    if (sched) {  // ---------------- schedule warp ----------------
         // The loop runs one copy of the 16-word schedule body for all six slices of a step (block-1
         // slices 1-3 of step i, then block-2 slices 1-3 of step i+1).  The rounds warp on the next
         // sub-partition slows down with the amount of distinct code this warp runs (per chain step,
@@ -422,15 +468,15 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
             for (int j = 9; j < 15; ++j) w[j] = 0;
             w[15] = 96u * 8u;
 #pragma unroll
-            for (int j = 0; j < 16; ++j) sm.kw2[buf][j][lane] = pk::kSha256K[j] + w[j];
+            for (int j = 0; j < 16; ++j) sm.kw2[buf][j][lane] = pk::add2<FS>(pk::kSha256K[j], w[j], one);
         };
         {
             uint32_t w[16];
             block2_head(0, 0, w);
 #pragma unroll 1
-            for (int q = 1; q < 4; ++q) schedule16(w, sm.kw2[0], q, lane);
+            for (int q = 1; q < 4; ++q) schedule16<FS>(w, sm.kw2[0], q, lane, one);
         }
-        bar_arrive(4);
+        bar_arrive(bar_b2);
 #pragma unroll 1
         for (int64_t i = 0; i < nmax; ++i) {
             if (i + 1 == nmax) pk::pdl_launch_dependents();
@@ -439,10 +485,10 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
 #pragma unroll
                 for (int j = 0; j < 8; ++j) w[j] = 0;  // k_{-1} = 0^32
             } else {
-                bar_sync(5);  // k_{i-1} published; the rounds warp has finished step i-1
+                bar_sync(bar_k);  // k_{i-1} published; the rounds warp has finished step i-1
 #pragma unroll
                 for (int j = 0; j < 8; ++j) w[j] = sm.kpub[j][lane];
-                bar_arrive(4);  // block-2 schedule of step i (made during the previous iteration)
+                bar_arrive(bar_b2);  // block-2 schedule of step i (made during the previous iteration)
             }
 #pragma unroll
             for (int j = 0; j < 8; ++j) w[8 + j] = dw[j];
@@ -451,11 +497,14 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
 #pragma unroll 1
             for (int sl = 1; sl <= slices; ++sl) {
                 if (sl == 4) block2_head(i + 1, buf, w);
-                schedule16(w, sl <= 3 ? sm.kw1 : sm.kw2[buf], sl <= 3 ? sl : sl - 3, lane);
-                // constant barrier ids (a run-time id reserves all 16 named barriers)
-                if (sl == 1) bar_arrive(1);
-                else if (sl == 2) bar_arrive(2);
-                else if (sl == 3) bar_arrive(3);
+                schedule16<FS>(w, sl <= 3 ? sm.kw1 : sm.kw2[buf], sl <= 3 ? sl : sl - 3, lane, one);
+                if (kPairs == 1) {  // constant barrier ids (a run-time id reserves all 16 named barriers)
+                    if (sl == 1) bar_arrive(1);
+                    else if (sl == 2) bar_arrive(2);
+                    else if (sl == 3) bar_arrive(3);
+                } else if (sl == 3) {
+                    bar_arrive(bar_s1);
+                }
             }
         }
         __syncthreads();  // stay resident until the rounds warp has consumed every phase
@@ -479,33 +528,64 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
             for (int j = 0; j < 8; ++j) pk::round_kw(a_, b_, c_, d_, e_, f_, g_, h_, kd[j]);
             v[0] = a_; v[1] = b_; v[2] = c_; v[3] = d_; v[4] = e_; v[5] = f_; v[6] = g_; v[7] = h_;
         }
-        bar_sync(1);
-        rounds16_kw(v, sm.kw1, 1, lane);
-        bar_sync(2);
-        rounds16_kw(v, sm.kw1, 2, lane);
-        bar_sync(3);
-        rounds16_kw(v, sm.kw1, 3, lane);
+        if (kPairs == 1) {
+            bar_sync(1);
+            rounds16_kw<pk::kAddsPlain>(v, sm.kw1, 1, lane, one);
+            bar_sync(2);
+            rounds16_kw<pk::kAddsPlain>(v, sm.kw1, 2, lane, one);
+            bar_sync(3);
+            rounds16_kw<pk::kAddsPlain>(v, sm.kw1, 3, lane, one);
+        } else {
+            bar_sync(bar_s1);
+            rounds16_kw<pk::kAddsPlain>(v, sm.kw1, 1, lane, one);
+            rounds16_kw<pk::kAddsPlain>(v, sm.kw1, 2, lane, one);
+            rounds16_kw<pk::kAddsPlain>(v, sm.kw1, 3, lane, one);
+        }
         uint32_t st[8] = {PK_IV0 + v[0], PK_IV1 + v[1], PK_IV2 + v[2], PK_IV3 + v[3],
                           PK_IV4 + v[4], PK_IV5 + v[5], PK_IV6 + v[6], PK_IV7 + v[7]};
-        bar_sync(4);  // block-2 schedule of step i
+        bar_sync(bar_b2);  // block-2 schedule of step i
         const uint32_t (*kw2)[kChainLanes] = sm.kw2[i & 1];
 #pragma unroll
         for (int j = 0; j < 8; ++j) v[j] = st[j];
 #pragma unroll 1
-        for (int q = 0; q < 4; ++q) rounds16_kw(v, kw2, q, lane);
+        for (int q = 0; q < 4; ++q) rounds16_kw<pk::kAddsPlain>(v, kw2, q, lane, one);
 #pragma unroll
         for (int j = 0; j < 8; ++j) p[j] = st[j] + v[j];
         if (i < n) store_digest(keys + 32ull * (a + i), p);
         if (i + 1 < nmax) {
 #pragma unroll
             for (int j = 0; j < 8; ++j) sm.kpub[j][lane] = p[j];
-            bar_arrive(5);
+            bar_arrive(bar_k);
         }
     }
     __syncthreads();
 }
 
 unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1) / block); }
+
+// Shared memory of the four-pair chain CTA: its four ChainSmem (100 KiB), padded past half of an SM's
+// shared memory so that no SM holds two of these CTAs (the launch becomes resident while the chunk digests
+// drain, and would otherwise stack CTAs on the SMs that free up first).
+constexpr size_t kChainPackedSmem = 116 * 1024;
+static_assert(kChainPackedSmem >= 4 * sizeof(ChainSmem), "four pairs fit");
+
+// Raise the four-pair chain CTA's shared-memory limit once per device.
+cudaError_t chain_packed_attr() {
+    static std::mutex mu;
+    static bool done[256] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 256) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!done[dev]) {
+        e = cudaFuncSetAttribute(k_chain<4, pk::kAddsFma>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kChainPackedSmem);
+        if (e != cudaSuccess) return e;
+        done[dev] = true;
+    }
+    return cudaSuccess;
+}
 
 }  // namespace
 
@@ -560,8 +640,19 @@ cudaError_t pk_launch_derive_enc(const pk_ctx *ctx, const int32_t *tokens, uint6
             : pk_launch(k_chunk_digest<pk::kAddsPlain>, grid, kDigestBlock, s, tokens, tok_off,
                         (const int64_t *)key_off, R, C, pad, keys, dw, one);
     if (e != cudaSuccess) return e;
-    e = pk_launch(k_chain, grid_for(R, kChainLanes), 2 * kChainLanes, s, (const int64_t *)key_off, desc_idx,
-                  (const uint8_t *)digests, R, D, keys);
+    // Chains: one pair per CTA while the groups of 32 requests fit one per SM; four pairs per CTA (one CTA
+    // per SM, each pair on its own sub-partition) for more groups.
+    const uint32_t groups = grid_for(R, kChainLanes);
+    if (ctx->sm_count == 0 || groups <= ctx->sm_count) {
+        e = pk_launch_smem(k_chain<1, pk::kAddsPlain>, groups, 2 * kChainLanes, sizeof(ChainSmem), s,
+                           (const int64_t *)key_off, desc_idx, (const uint8_t *)digests, R, D, keys, groups, one);
+    } else {
+        e = chain_packed_attr();
+        const uint32_t grid = groups <= 4 * ctx->sm_count ? ctx->sm_count : grid_for(groups, 4);
+        if (e == cudaSuccess)
+            e = pk_launch_smem(k_chain<4, pk::kAddsFma>, grid, 8 * kChainLanes, kChainPackedSmem, s,
+                               (const int64_t *)key_off, desc_idx, (const uint8_t *)digests, R, D, keys, groups, one);
+    }
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

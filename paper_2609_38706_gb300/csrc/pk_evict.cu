@@ -64,12 +64,22 @@ __device__ __forceinline__ unsigned int ld_acquire(const unsigned int *p) {
     return v;
 }
 
+// The bound of a launch's barrier waits, and the CTA that withholds its
+// arrival at the first barrier (none in a normal launch; the timeout test
+// names one, so that the others' waits run out).
+struct BarrierBound {
+    uint32_t spin_limit;
+    uint32_t withheld_cta;
+};
+
 // Grid-wide barrier with a bounded wait.  Returns false (in every thread of
 // the CTA) when the wait gave up; the status word then holds PK_ERR_TIMEOUT.
-__device__ bool grid_sync(EvictHeader *h, int32_t *status) {
+// A withheld CTA returns false without arriving.
+__device__ bool grid_sync(EvictHeader *h, int32_t *status, const BarrierBound &bb) {
     __shared__ int ok;
     __syncthreads();
-    if (threadIdx.x == 0) {
+    if (threadIdx.x == 0 && blockIdx.x == bb.withheld_cta) ok = 0;
+    if (threadIdx.x == 0 && blockIdx.x != bb.withheld_cta) {
         ok = 1;
         const unsigned int g = ld_acquire(&h->gen);
         __threadfence();
@@ -80,7 +90,7 @@ __device__ bool grid_sync(EvictHeader *h, int32_t *status) {
         } else {
             uint32_t it = 0;
             while (ld_acquire(&h->gen) == g) {
-                if (++it > kSpinLimit) {
+                if (++it > bb.spin_limit) {
                     ok = 0;
                     pk::set_status(status, PK_ERR_TIMEOUT);
                     break;
@@ -284,7 +294,7 @@ __global__ void __launch_bounds__(kEvThreads, 1)
 k_evict(pk_entry *table, unsigned long long *stamps, uint64_t capacity, unsigned long long *counter, uint64_t budget,
         uint64_t keep, EvictHeader *h, uint32_t *bitmap, uint32_t *evbm, uint8_t *dist, unsigned long long *list,
         uint32_t *list_slot, uint32_t *evicted, uint64_t evicted_cap, unsigned long long *n_evicted_out,
-        int32_t *status) {
+        int32_t *status, BarrierBound bb) {
     __shared__ unsigned int sh_hist[256];
     __shared__ unsigned long long sh_sel[2];
     __shared__ unsigned long long sh_removed;
@@ -369,7 +379,7 @@ k_evict(pk_entry *table, unsigned long long *stamps, uint64_t capacity, unsigned
         atomicMax(&h->inv_min, ~lo);
         atomicMax(&h->max, hi);
     }
-    if (!grid_sync(h, status)) return;
+    if (!grid_sync(h, status, bb)) return;
     const unsigned long long n = __ldcg(&h->n);
     unsigned long long prefix_v = 0;  // v, once selected
 
@@ -403,7 +413,7 @@ k_evict(pk_entry *table, unsigned long long *stamps, uint64_t capacity, unsigned
             __syncthreads();
             for (uint32_t b = tid; b < 256; b += blockDim.x)
                 if (sh_hist[b]) atomicAdd(&h->hist[p][b], sh_hist[b]);
-            if (!grid_sync(h, status)) return;
+            if (!grid_sync(h, status, bb)) return;
             if (tid < 32) {  // bucket holding `rank`: 8 buckets per lane, then a warp scan
                 unsigned long long c[8], sum = 0;
 #pragma unroll
@@ -483,7 +493,7 @@ k_evict(pk_entry *table, unsigned long long *stamps, uint64_t capacity, unsigned
             }
         }
     }
-    if (!grid_sync(h, status)) return;
+    if (!grid_sync(h, status, bb)) return;
     if (n > keep) {
         // 4c. compaction: one thread per bitmap word, for the clusters that start in it.  Clusters
         // that end within the 64 positions of the word and the next one are planned in registers
@@ -590,7 +600,7 @@ k_evict(pk_entry *table, unsigned long long *stamps, uint64_t capacity, unsigned
             }
         }
     }
-    if (!grid_sync(h, status)) return;
+    if (!grid_sync(h, status, bb)) return;
     if (gtid == 0 && n_evicted_out) *n_evicted_out = __ldcg(&h->n_evicted);
 }
 
@@ -619,7 +629,8 @@ static cudaError_t evict_resident(int dev, uint64_t *out) {
 }
 
 cudaError_t pk_launch_evict(const pk_ctx *ctx, uint64_t budget, uint64_t keep, void *scratch, uint32_t *evicted,
-                            uint64_t evicted_cap, unsigned long long *n_evicted, int32_t *status, cudaStream_t s) {
+                            uint64_t evicted_cap, unsigned long long *n_evicted, int32_t *status, cudaStream_t s,
+                            uint32_t spin_limit, bool withhold_first_cta) {
     int dev = 0;
     uint64_t resident = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -648,7 +659,9 @@ cudaError_t pk_launch_evict(const pk_ctx *ctx, uint64_t budget, uint64_t keep, v
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    const BarrierBound bb{spin_limit == 0 || spin_limit > kSpinLimit ? kSpinLimit : spin_limit,
+                          withhold_first_cta ? 0u : 0xffffffffu};
     e = cudaLaunchKernelEx(&cfg, k_evict, ctx->table, ctx->stamps, ctx->capacity, ctx->counter_dev, budget, keep, h,
-                           bitmap, evbm, dist, list, list_slot, evicted, evicted_cap, n_evicted, status);
+                           bitmap, evbm, dist, list, list_slot, evicted, evicted_cap, n_evicted, status, bb);
     return e != cudaSuccess ? e : cudaGetLastError();
 }

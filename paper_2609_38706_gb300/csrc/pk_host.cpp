@@ -403,6 +403,15 @@ int pk_evict(pk_ctx *ctx, uint64_t budget, uint64_t keep, void *scratch_dev, siz
                                    reinterpret_cast<cudaStream_t>(stream)));
 }
 
+int pk_evict_barrier_timeout_test(pk_ctx *ctx, uint64_t budget, void *scratch_dev, size_t scratch_bytes,
+                                  uint32_t spin_limit, int32_t *status_dev, pk_stream stream) {
+    if (!ctx || !ctx->stamps || !scratch_dev || !aligned16(scratch_dev) || !status_dev || spin_limit == 0)
+        return PK_ERR_ARG;
+    if (scratch_bytes < pk_evict_scratch_bytes_impl(ctx->capacity) || !aligned(status_dev, 4)) return PK_ERR_ARG;
+    return cuda_rc(pk_launch_evict(ctx, budget, budget, scratch_dev, nullptr, 0, nullptr, status_dev,
+                                   reinterpret_cast<cudaStream_t>(stream), spin_limit, true));
+}
+
 int pk_key_string(const uint8_t key16[16], char out[22]) {
     if (!key16 || !out) return PK_ERR_ARG;
     base64_16(key16, out);

@@ -28,7 +28,8 @@ struct pk_ctx {
     uint64_t capacity;
     pk_entry *table;
     unsigned long long *counter_dev;  // [0] entries in the table; [1] requests handed out by a lookup-and-store;
-                                      // [2] entries deferred in a store call; [3] keys its admit kernel claimed
+                                      // [2] entries deferred in a store call; [3], [4] keys its claim and admit
+                                      // kernels claimed (folded into [0] by its finalize kernel)
     unsigned long long epoch;         // last store call number
     unsigned long long *stamps;       // budget mode: last-use stamp per entry (pk_attach_stamps), else NULL
     uint32_t pad_kw[64];              // K_t + W_t of a chunk's final (padding-only) block, C % 16 == 0
@@ -73,8 +74,12 @@ cudaError_t pk_launch_compare_pages(const uint32_t *slots, const uint8_t *pages,
                                     uint64_t n_ref, uint64_t page_bytes, int32_t *verdict, unsigned long long *counts,
                                     int32_t *status, cudaStream_t s);
 uint64_t pk_evict_scratch_bytes_impl(uint64_t capacity);
+// spin_limit: polls of a barrier wait before it gives up (0 = the default of
+// about a second); withhold_first_cta: CTA 0 does not arrive at the first
+// barrier (the timeout test).
 cudaError_t pk_launch_evict(const pk_ctx *ctx, uint64_t budget, uint64_t keep, void *scratch, uint32_t *evicted,
-                            uint64_t evicted_cap, unsigned long long *n_evicted, int32_t *status, cudaStream_t s);
+                            uint64_t evicted_cap, unsigned long long *n_evicted, int32_t *status, cudaStream_t s,
+                            uint32_t spin_limit = 0, bool withhold_first_cta = false);
 cudaError_t pk_launch_key_strings(const uint8_t *keys, uint64_t n, const uint8_t *prefix, uint32_t plen,
                                   uint32_t width, uint8_t *out, cudaStream_t s);
 cudaError_t pk_launch_lookup_store(const pk_ctx *ctx, unsigned long long epoch, const uint8_t *keys,
@@ -92,6 +97,22 @@ static inline cudaError_t pk_launch(void (*kernel)(KArgs...), unsigned grid, uns
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(block);
     cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+// The same with dynamic shared memory.
+template <typename... KArgs, typename... Args>
+static inline cudaError_t pk_launch_smem(void (*kernel)(KArgs...), unsigned grid, unsigned block, size_t smem,
+                                         cudaStream_t s, Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(block);
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

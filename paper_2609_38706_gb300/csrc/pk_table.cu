@@ -364,10 +364,10 @@ k_first_miss(const int64_t *key_off, uint32_t R, uint64_t key_capacity,
 //   key absent: in claim mode, CAS the key into the first empty entry (then
 //   bid, PENDING); in defer mode, leave the entry DEFERRED for the admit
 //   kernel and write nothing
-// A warp takes claim mode when the entry count it reads plus the call's
+// The call takes claim mode when the entry count at its start plus its
 // entries stays below capacity: the whole call fits, so no key is refused.
-// (A warp that reads the count after other blocks added their claims may
-// take defer mode; its deferred keys then all fit as well.)
+// The count is read from a word no kernel of the call changes, so every warp
+// takes the same mode.
 // Admit kernel: nothing to do unless entries were deferred.  If the deferred
 // entries fit in the room left (capacity - 1 - count), all are claimed in
 // parallel; otherwise one CTA walks the deferred entries in index order,
@@ -379,10 +379,12 @@ k_first_miss(const int64_t *key_off, uint32_t R, uint64_t key_capacity,
 // once every claim is in: the lowest claimant is INSERTED, the others
 // PRESENT with its slot.
 //
-// Context counter words: [0] entries in the table, [1] requests handed out
-// by a work-taking lookup-and-store, [2] entries deferred in this call,
-// [3] keys claimed by the admit kernel in this call (added to [0] and
-// cleared with [2] by the finalize kernel).
+// Context counter words: [0] entries in the table at the start of the call
+// (constant while its claim and admit kernels run, so that every warp takes
+// the same mode), [1] requests handed out by a work-taking lookup-and-store,
+// [2] entries deferred in this call, [3] keys the claim kernel claimed,
+// [4] keys the admit kernel claimed; the finalize kernel adds [3] and [4] to
+// [0] and clears [2..4].
 // ---------------------------------------------------------------------------
 enum Examine { kAdvance, kDone, kClaimedHere };
 enum ClaimMode : uint32_t {
@@ -484,8 +486,9 @@ struct ClaimCtx {
     unsigned long long *stamps;  // budget mode: last-use stamp per entry, else NULL
 };
 
-// Mode of a claim kernel's warp: claim when the entry count plus the call's
-// entries stays below capacity (the whole call fits), else defer.
+// Mode of a claim kernel's warp: claim when the entry count at the start of
+// the call plus the call's entries stays below capacity (the whole call
+// fits), else defer.
 __device__ __forceinline__ uint32_t claim_mode(const unsigned long long *counter, uint64_t n, uint64_t capacity) {
     unsigned long long cnt = 0;
     if ((threadIdx.x & 31) == 0) cnt = ld_volatile_u64(counter);
@@ -636,7 +639,7 @@ __device__ __forceinline__ bool in_store_range(const int64_t *key_off, const int
 }
 
 // Adds the warp's claims and deferred entries to the block totals, then the
-// block totals to counter[0] (entries) and counter[2] (deferred): one atomic
+// block totals to counter[3] (claims) and counter[2] (deferred): one atomic
 // per block and word (same-address atomics serialise in L2).
 __device__ __forceinline__ void count_claims(unsigned long long *block_sums, uint32_t claims, uint32_t deferred,
                                              unsigned long long *counter) {
@@ -645,7 +648,7 @@ __device__ __forceinline__ void count_claims(unsigned long long *block_sums, uin
     if ((threadIdx.x & 31) == 0 && w) atomicAdd_block(block_sums, (unsigned long long)w);
     if ((threadIdx.x & 31) == 0 && d) atomicAdd_block(block_sums + 1, (unsigned long long)d);
     __syncthreads();
-    if (threadIdx.x == 0 && block_sums[0]) atomicAdd(counter, block_sums[0]);
+    if (threadIdx.x == 0 && block_sums[0]) atomicAdd(counter + 3, block_sums[0]);
     if (threadIdx.x == 0 && block_sums[1]) atomicAdd(counter + 2, block_sums[1]);
 }
 
@@ -998,8 +1001,9 @@ __device__ __forceinline__ void admit_write(uint64_t e, int32_t res, uint32_t ou
 
 // Store, admit kernel (see the store comment above).  The call's entries are
 // [0, n), or [0, min(n, key_off[R])) in range and lookup-and-store mode;
-// counter[0] is the entry count after the claim kernel, counter[2] the
-// number of DEFERRED entries; keys claimed here are added to counter[3].
+// counter[0] + counter[3] is the entry count after the claim kernel,
+// counter[2] the number of DEFERRED entries; keys claimed here are added to
+// counter[4].
 // Within the call the entry count can only reach capacity - 1: the claim
 // kernel claims only when the whole call fits, and here at most `room` keys
 // are claimed.
@@ -1012,7 +1016,7 @@ __device__ __forceinline__ void store_admit(pk_entry *table, uint64_t mask, uint
     __shared__ unsigned long long s_claims;
     const unsigned long long deferred = __ldcg(counter + 2);
     if (deferred == 0) return;  // every key was decided by the claim kernel
-    const unsigned long long count = __ldcg(counter);
+    const unsigned long long count = __ldcg(counter) + __ldcg(counter + 3);
     const unsigned long long room = count + 1 < capacity ? capacity - 1 - count : 0ull;
     uint64_t end = n;
     if (key_off) {
@@ -1042,7 +1046,7 @@ __device__ __forceinline__ void store_admit(pk_entry *table, uint64_t mask, uint
         const uint32_t wc = __reduce_add_sync(kFull, claims);
         if (lane == 0 && wc) atomicAdd_block(&s_claims, (unsigned long long)wc);
         __syncthreads();
-        if (threadIdx.x == 0 && s_claims) atomicAdd(counter + 3, s_claims);
+        if (threadIdx.x == 0 && s_claims) atomicAdd(counter + 4, s_claims);
         return;
     }
     // More deferred entries than room: one CTA walks them in index order, 256
@@ -1085,7 +1089,7 @@ __device__ __forceinline__ void store_admit(pk_entry *table, uint64_t mask, uint
             __syncthreads();  // s_warp and s_claims are rewritten next round
         }
     }
-    if (threadIdx.x == 0 && admitted) atomicAdd(counter + 3, admitted);
+    if (threadIdx.x == 0 && admitted) atomicAdd(counter + 4, admitted);
 }
 
 __global__ void __launch_bounds__(256)
@@ -1101,18 +1105,22 @@ k_store_admit(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
 // Store, last kernel: each PENDING entry reads its key's slot/owner word,
 // final once every claim is in: the lowest claimant is INSERTED, the others
 // PRESENT with its slot.  In range mode, entries past key_off[R] (not keys
-// of this batch) are skipped.  The admit kernel's claims are added to the
-// entry count, and the call's counter words [2] and [3] cleared.
+// of this batch) are skipped.  The call's claims are added to the entry
+// count, and its counter words [2..4] cleared.
 __global__ void __launch_bounds__(256)
 k_store_finalize(const pk_entry *table, uint64_t n, const int64_t *key_off, uint32_t R,
                  int32_t *result, uint32_t *slot_out, unsigned long long *counter) {
     pk::pdl_launch_dependents();
     pk::pdl_wait(table, key_off, result, slot_out, counter);
     const uint64_t e = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (e == 0 && __ldcg(counter + 2)) {
-        counter[0] += __ldcg(counter + 3);
-        counter[2] = 0;
-        counter[3] = 0;
+    if (e == 0) {
+        const unsigned long long c2 = __ldcg(counter + 2), c3 = __ldcg(counter + 3), c4 = __ldcg(counter + 4);
+        if (c3 | c4) counter[0] += c3 + c4;
+        if (c2 | c3 | c4) {
+            counter[2] = 0;
+            counter[3] = 0;
+            counter[4] = 0;
+        }
     }
     if (e >= n) return;
     if (key_off && (int64_t)e >= (R > 0 ? __ldcg(key_off + R) : 0)) {
@@ -1171,11 +1179,11 @@ __global__ void k_mark_loaded(pk_entry *table, uint64_t capacity) {
 // positions live in this one file-scope array, shared by every call.
 // ---------------------------------------------------------------------------
 struct NoallocScratch {
-    // [0] entries in the table (set by the scan, then claims), [1] largest
-    // call number found in the table, [2] entries deferred in this call,
-    // [3] keys its admit kernel claimed: [0], [2] and [3] are the words a
-    // context's counter holds at the same indices
-    unsigned long long word[4];
+    // [0] entries in the table (set by the scan), [1] largest call number
+    // found in the table, [2] entries deferred in this call, [3] keys its
+    // claim kernel claimed, [4] keys its admit kernel claimed: [0] and [2..4]
+    // are the words a context's counter holds at the same indices
+    unsigned long long word[5];
     uint32_t pos[PK_NOALLOC_MAX_ENTRIES];  // table position of each PENDING entry
 };
 static __device__ __align__(256) NoallocScratch g_noalloc_scratch;
@@ -1451,7 +1459,7 @@ cudaError_t pk_launch_store_noalloc(pk_entry *table, uint32_t capacity_log2, uin
     if (!sc) return cudaErrorInvalidSymbol;
     if (n == 0) return cudaSuccess;
     const uint64_t capacity = 1ull << capacity_log2;
-    // the four counter words must start at zero; pos needs no clearing
+    // the five counter words must start at zero; pos needs no clearing
     e = cudaMemsetAsync(sc, 0, sizeof sc->word, s);
     if (e != cudaSuccess) return e;
     const uint64_t scan_blocks = (capacity + 255) / 256;

@@ -111,6 +111,7 @@ def lib() -> ctypes.CDLL:
             "pk_attach_stamps": (ctypes.c_int, [_VP, _VP, ctypes.c_size_t, _VP]),
             "pk_evict_scratch_bytes": (ctypes.c_size_t, [_U32]),
             "pk_evict": (ctypes.c_int, [_VP, _U64, _U64, _VP, ctypes.c_size_t, _VP, _U64, _VP, _VP, _VP]),
+            "pk_evict_barrier_timeout_test": (ctypes.c_int, [_VP, _U64, _VP, ctypes.c_size_t, _U32, _VP, _VP]),
             "pk_key_string": (ctypes.c_int, [_VP, _VP]),
             "pk_model_tag": (ctypes.c_int, [ctypes.POINTER(pk_descriptor), _VP]),
             "pk_key_strings": (ctypes.c_int, [_VP, _U64, _VP, _U32, _U32, _VP, _VP]),
@@ -420,6 +421,14 @@ def pk_evict(ctx: int, budget: int, keep: int, scratch: torch.Tensor, evicted: O
     _check(lib().pk_evict(ctx, budget, keep, _p(scratch), scratch.numel(), _p(evicted),
                           0 if evicted is None else evicted.numel(), _p(n_evicted), _p(status), _s(stream)),
            "pk_evict")
+
+
+def pk_evict_barrier_timeout_test(ctx: int, budget: int, scratch: torch.Tensor, spin_limit: int,
+                                  status: torch.Tensor, stream=None) -> None:
+    """Test hook: pk_evict with CTA 0 withholding its first barrier arrival and
+    the waits bounded at spin_limit polls (the status must end PK_ERR_TIMEOUT)."""
+    _check(lib().pk_evict_barrier_timeout_test(ctx, budget, _p(scratch), scratch.numel(), spin_limit, _p(status),
+                                               _s(stream)), "pk_evict_barrier_timeout_test")
 
 
 def pk_key_string(key16: bytes) -> str:

@@ -4,6 +4,8 @@ triples of the table, and after every eviction the removed slots, the entry
 count and the lookups of every key, bit-exact.  Positions are not compared
 (the compaction moves kept entries; only reachability is required, and the
 lookups check it)."""
+import time
+
 import numpy as np
 import pytest
 import torch
@@ -242,4 +244,37 @@ def test_large_table_sampled():
     run_evict(kt, bt, 500_000, 200_000)
     assert triples(kt) == bt.triples()
     check_lookups(kt, bt, np.ascontiguousarray(keys[rng.integers(0, 600_000, 20_000)]))
+    kt.close()
+
+
+def test_barrier_wait_runs_out_and_the_context_stays_usable():
+    """The bounded grid barrier of pk_evict: one CTA withholds its arrival at
+    the first barrier (a flag that nothing sets), the other CTAs' waits run
+    out after a short bound, the launch ends by itself with PK_ERR_TIMEOUT,
+    the table and stamps are untouched (the first barrier precedes every
+    write), and the next calls on the context work and match the oracle."""
+    from paper_2609_38706_gb300 import pk
+    from paper_2609_38706_gb300.service import KeyTable
+    log2 = 14
+    rng = np.random.default_rng(11)
+    pool = _keys(rng, 6000)
+    kt = KeyTable(16, log2)
+    kt.attach_stamps()
+    bt = O.BudgetTable(1 << log2)
+    sl = np.arange(pool.shape[0], dtype=np.uint32)
+    kt.store(torch.from_numpy(pool).cuda(), sl)
+    bt.store(pool, sl)
+    torch.cuda.synchronize()
+    kt.check("store")
+    table0, stamps0 = kt.table.clone(), kt.stamps.clone()
+    t0 = time.perf_counter()
+    pk.pk_evict_barrier_timeout_test(kt.ctx, 4000, kt.evict_scratch, 1 << 12, kt.status)
+    torch.cuda.synchronize()
+    took = time.perf_counter() - t0
+    assert kt.take_status() == pk.PK_ERR_TIMEOUT
+    assert took < 5.0
+    assert torch.equal(kt.table, table0) and torch.equal(kt.stamps, stamps0)
+    run_evict(kt, bt, 4000, 3000)  # the same eviction, now with every CTA arriving
+    assert triples(kt) == bt.triples()
+    check_lookups(kt, bt, pool)
     kt.close()
