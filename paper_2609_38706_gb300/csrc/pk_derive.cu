@@ -96,8 +96,12 @@ k_chunk_offsets(const int64_t *tok_off, uint32_t R, uint64_t n_tokens, uint32_t 
             n[j] = 0;
             if (r < R) {
                 const int64_t a = tok_off[r], b = tok_off[r + 1];
-                if (a < 0 || b < a || (uint64_t)b > n_tokens || desc_idx[r] >= D) bad = true;
-                else n[j] = (b - a) / C;
+                if (a < 0 || b < a || (uint64_t)b > n_tokens || desc_idx[r] >= D) {
+                    bad = true;
+                } else {  // 32-bit division when the request fits (64-bit division is a long library sequence)
+                    const uint64_t len = (uint64_t)(b - a);
+                    n[j] = len >> 32 ? (long long)(len / C) : (long long)((uint32_t)len / C);
+                }
             }
             local += n[j];
         }
