@@ -884,8 +884,10 @@ __device__ __forceinline__ uint64_t take_request(unsigned long long *tickets) {
 // resident CTAs whose warps take requests one at a time until none is left
 // (kTake true, for batches of more requests than resident warps: a warp done
 // with its request does not wait for the slowest request of its block).
+constexpr unsigned kLsBlock = 128;  // 72 registers: 7 CTAs (28 warps) per SM, against 3 CTAs (24 warps) of 256
+
 template <bool kTake>
-__global__ void __launch_bounds__(256, 3)
+__global__ void __launch_bounds__(kLsBlock, 7)
 k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
                    unsigned long long *counter, unsigned long long epoch, unsigned long long *stamps, const uint8_t *keys,
                    const uint32_t *new_slots, const int64_t *key_off, uint32_t R,
@@ -1302,7 +1304,7 @@ cudaError_t lookup_store_resident(uint64_t *out) {
     if (!cache[dev]) {
         int sms = 0, per_sm = 0;
         e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_lookup_store_req<true>, 256, 0);
+        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_lookup_store_req<true>, kLsBlock, 0);
         if (e != cudaSuccess) return e;
         cache[dev] = (uint64_t)sms * (uint64_t)(per_sm < 1 ? 1 : per_sm);
     }
@@ -1386,14 +1388,14 @@ cudaError_t pk_launch_lookup_store(const pk_ctx *ctx, unsigned long long epoch, 
         e = lookup_store_resident(&resident);
         if (e != cudaSuccess) return e;
         unsigned long long *tickets = ctx->counter_dev + 1;
-        if (R > 32 * resident) {  // more requests than resident warps: warps take requests as they finish
+        if (R > (kLsBlock / 32) * resident) {  // more requests than resident warps: warps take requests as they finish
             e = cudaMemsetAsync(tickets, 0, sizeof *tickets, s);
             if (e == cudaSuccess)
-                e = pk_launch(k_lookup_store_req<true>, (unsigned)resident, 256, s, ctx->table, mask, ctx->max_probe,
+                e = pk_launch(k_lookup_store_req<true>, (unsigned)resident, kLsBlock, s, ctx->table, mask, ctx->max_probe,
                               ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, new_slots, key_off, R,
                               key_capacity, slots, hit_chunks, result, slot_out, status, tickets);
         } else {
-            e = pk_launch(k_lookup_store_req<false>, grid_for(32ull * R, 256), 256, s, ctx->table, mask,
+            e = pk_launch(k_lookup_store_req<false>, grid_for(32ull * R, kLsBlock), kLsBlock, s, ctx->table, mask,
                           ctx->max_probe, ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, new_slots, key_off,
                           R, key_capacity, slots, hit_chunks, result, slot_out, status, tickets);
         }
