@@ -566,9 +566,9 @@ def main():
                                    "ms_per_step": e2e_inplace_total / args.steps,
                                    "note": "all inputs read by the kernels from pinned host memory"}},
         # per step: chunk offsets, chunk+descriptor digests, chain; lookup-and-store (one kernel of
-        # request warps, or per key + per-request tail for few long requests); admit; finalize
+        # request warps, or per key + per-request tail for few long requests); finalize
         "critical_path": critical_path(wl, derive_s, peaks),
-        "gpu_launches": (3 + (1 if (R >= 1024 or N_cap <= 64 * R) else 2) + 2) * args.steps,
+        "gpu_launches": (3 + (1 if (R >= 1024 or N_cap <= 64 * R) else 2) + 1) * args.steps,
         "clocks": clk,
     }
     # Store-side omission test (comparison step, pk_compare_pages): 16,384 joined pages of 16 KiB against a

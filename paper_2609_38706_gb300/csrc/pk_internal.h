@@ -28,8 +28,9 @@ struct pk_ctx {
     uint64_t capacity;
     pk_entry *table;
     unsigned long long *counter_dev;  // [0] entries in the table; [1] requests handed out by a lookup-and-store;
-                                      // [2] entries deferred in a store call; [3], [4] keys its claim and admit
-                                      // kernels claimed (folded into [0] by its finalize kernel)
+                                      // [2] entries deferred in a store call; [3], [4] keys its claims and its
+                                      // admission pass claimed (folded into [0] by its finalize kernel); [5] CTAs
+                                      // of its claim kernel done
     unsigned long long epoch;         // last store call number
     unsigned long long *stamps;       // budget mode: last-use stamp per entry (pk_attach_stamps), else NULL
     uint32_t pad_kw[64];              // K_t + W_t of a chunk's final (padding-only) block, C % 16 == 0
@@ -38,7 +39,7 @@ struct pk_ctx {
 
 // internal per-entry states between the store kernels (never returned)
 #define PK_STORE_PENDING 0x40000000   /* claimed or bid: the finalize kernel decides */
-#define PK_STORE_DEFERRED 0x40000001  /* absent, left to the admit kernel */
+#define PK_STORE_DEFERRED 0x40000001  /* absent, left to the admission pass */
 
 // Launchers (pk_derive.cu, pk_table.cu).  Each returns the launch error.
 cudaError_t pk_launch_digest_descriptors(const uint8_t *enc, uint64_t enc_bytes, const int64_t *enc_off,

@@ -362,29 +362,32 @@ k_first_miss(const int64_t *key_off, uint32_t R, uint64_t key_capacity,
 //   key claimed in this call (by anyone): bid (~index, slot) on the entry's
 //   slot/owner word and leave PENDING with the entry position
 //   key absent: in claim mode, CAS the key into the first empty entry (then
-//   bid, PENDING); in defer mode, leave the entry DEFERRED for the admit
-//   kernel and write nothing
+//   bid, PENDING); in defer mode, leave the entry DEFERRED for the admission
+//   pass and write nothing
 // The call takes claim mode when the entry count at its start plus its
 // entries stays below capacity: the whole call fits, so no key is refused.
 // The count is read from a word no kernel of the call changes, so every warp
 // takes the same mode.
-// Admit kernel: nothing to do unless entries were deferred.  If the deferred
-// entries fit in the room left (capacity - 1 - count), all are claimed in
-// parallel; otherwise one CTA walks the deferred entries in index order,
-// each round letting at most `room` of them claim (so at most `room` new
-// keys), until the room is gone; the rest are bids on keys this call already
-// claimed, or TABLE_FULL.  That is exactly the sequential rule: the first
-// `room` distinct new keys (by lowest index) go in, later ones are refused.
+// Admission pass, by the claim kernel's last CTA to finish: nothing to do
+// unless entries were deferred (a call that may not fit: rare, and then one
+// CTA's work).  If the deferred entries fit in the room left (capacity - 1 -
+// count), all are claimed; otherwise the CTA walks the deferred entries in
+// index order, each round letting at most `room` of them claim (so at most
+// `room` new keys), until the room is gone; the rest are bids on keys this
+// call already claimed, or TABLE_FULL.  That is exactly the sequential rule:
+// the first `room` distinct new keys (by lowest index) go in, later ones are
+// refused.  (A separate launch for this pass cost about 2.5 us on every
+// store call.)
 // Finalize kernel: each PENDING entry reads its key's slot/owner word, final
 // once every claim is in: the lowest claimant is INSERTED, the others
 // PRESENT with its slot.
 //
 // Context counter words: [0] entries in the table at the start of the call
-// (constant while its claim and admit kernels run, so that every warp takes
-// the same mode), [1] requests handed out by a work-taking lookup-and-store,
-// [2] entries deferred in this call, [3] keys the claim kernel claimed,
-// [4] keys the admit kernel claimed; the finalize kernel adds [3] and [4] to
-// [0] and clears [2..4].
+// (constant while its claim kernel runs, so that every warp takes the same
+// mode), [1] requests handed out by a work-taking lookup-and-store, [2]
+// entries deferred in this call, [3] keys its claims claimed, [4] keys its
+// admission pass claimed, [5] CTAs of the claim kernel done (reset by the
+// last); the finalize kernel adds [3] and [4] to [0] and clears [2..4].
 // ---------------------------------------------------------------------------
 enum Examine { kAdvance, kDone, kClaimedHere };
 enum ClaimMode : uint32_t {
@@ -450,7 +453,7 @@ __device__ __forceinline__ Examine examine(pk_entry *ent, uint64_t pos, uint4 cu
             out = PK_NO_SLOT;
             return kDone;
         }
-        if (mode != kModeClaim) {  // absent: left to the admit kernel, or refused
+        if (mode != kModeClaim) {  // absent: left to the admission pass, or refused
             res = mode == kModeDefer ? PK_STORE_DEFERRED : PK_ERR_TABLE_FULL;
             out = PK_NO_SLOT;
             return kDone;
@@ -652,6 +655,135 @@ __device__ __forceinline__ void count_claims(unsigned long long *block_sums, uin
     if (threadIdx.x == 0 && block_sums[1]) atomicAdd(counter + 2, block_sums[1]);
 }
 
+// Result of a deferred entry decided by the admission pass.  pos_out: where a
+// PENDING entry's table position goes (slot_out for a context; the
+// allocation-free store keeps positions apart and writes PK_NO_SLOT to
+// slot_out).
+__device__ __forceinline__ void admit_write(uint64_t e, int32_t res, uint32_t out, int32_t *result,
+                                            uint32_t *slot_out, uint32_t *pos_out, int32_t *status) {
+    result[e] = res;
+    if (res == PK_STORE_PENDING && pos_out != slot_out) {
+        pos_out[e] = out;
+        slot_out[e] = PK_NO_SLOT;
+    } else {
+        slot_out[e] = out;
+    }
+    if (res < 0) set_status(status, res);
+}
+
+// Store, admission pass (see the store comment above), run by one CTA: the
+// last CTA of the claim kernel to finish.  The call's entries are [0, n), or
+// [0, min(n, key_off[R])) in range and lookup-and-store mode; counter[0] +
+// counter[3] is the entry count after the claims, counter[2] the number of
+// DEFERRED entries; keys claimed here are added to counter[4].  Within the
+// call the entry count can only reach capacity - 1: the claim kernel claims
+// only when the whole call fits, and here at most `room` keys are claimed.
+// Out of line: the claim kernels' registers stay those of their main loops.
+__device__ __noinline__ void store_admit(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
+                                            unsigned long long *counter, unsigned long long epoch,
+                                            unsigned long long *stamps, const uint8_t *keys, const uint32_t *slots,
+                                            uint64_t n, const int64_t *key_off, uint32_t R, int32_t *result,
+                                            uint32_t *slot_out, uint32_t *pos_out, int32_t *status) {
+    __shared__ uint32_t s_warp[8];
+    __shared__ unsigned long long s_claims;
+    const unsigned long long deferred = __ldcg(counter + 2);
+    if (deferred == 0) return;  // every key was decided by the claim kernel
+    const unsigned long long count = __ldcg(counter) + __ldcg(counter + 3);
+    const unsigned long long room = count + 1 < capacity ? capacity - 1 - count : 0ull;
+    uint64_t end = n;
+    if (key_off) {
+        const int64_t t = R ? __ldcg(key_off + R) : 0;
+        if (t < (int64_t)end) end = t > 0 ? (uint64_t)t : 0;
+    }
+    const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (deferred <= room) {
+        // At most `deferred` distinct keys: all fit.  Claimed by all warps of the CTA at once.
+        const ClaimCtx c{table, mask, max_probe, epoch, kModeClaim, stamps};
+        uint32_t claims = 0;
+        if (threadIdx.x == 0) s_claims = 0;
+        __syncthreads();
+        for (uint64_t base = 32 * warp; base < end; base += blockDim.x) {  // uniform per warp
+            const uint64_t e = base + lane;
+            ProbeKey s;
+            s.pending = false;
+            if (e < end && __ldcg(result + e) == PK_STORE_DEFERRED)
+                probe_start(s, ld_cg_v4(keys + 32 * e), e, mask, __ldcg(slots + e));
+            const bool mine = s.pending;
+            int32_t res;
+            uint32_t out, lslot;
+            warp_claim<false>(c, s, res, out, lslot, claims);
+            if (mine) admit_write(e, res, out, result, slot_out, pos_out, status);
+        }
+        const uint32_t wc = __reduce_add_sync(kFull, claims);
+        if (lane == 0 && wc) atomicAdd_block(&s_claims, (unsigned long long)wc);
+        __syncthreads();
+        if (threadIdx.x == 0 && s_claims) atomicAdd(counter + 4, s_claims);
+        return;
+    }
+    // More deferred entries than room: walk them in index order, one tile of
+    // blockDim.x at a time.  Each round the first `left` undecided entries of
+    // the tile (at most `left` distinct keys) claim or bid; once the room is
+    // gone the rest only bid on keys this call claimed, or are refused.  Every
+    // round decides at least one entry.
+    unsigned long long left = room, admitted = 0;
+    for (uint64_t base = 0; base < end; base += blockDim.x) {
+        const uint64_t e = base + threadIdx.x;
+        bool pend = e < end && __ldcg(result + e) == PK_STORE_DEFERRED;
+        const uint4 key = pend ? ld_cg_v4(keys + 32 * e) : make_uint4(0, 0, 0, 0);
+        const uint32_t sl = pend ? __ldcg(slots + e) : 0u;
+        for (;;) {
+            const uint32_t ball = __ballot_sync(kFull, pend);
+            if (lane == 0) s_warp[warp] = __popc(ball);
+            if (threadIdx.x == 0) s_claims = 0;
+            if (__syncthreads_count(pend) == 0) break;  // the tile is decided (uniform)
+            uint32_t rank = __popc(ball & lanemask_lt());
+            for (uint32_t w = 0; w < warp; ++w) rank += s_warp[w];
+            const bool act = pend && (left == 0 || rank < left);
+            const ClaimCtx c{table, mask, max_probe, epoch, left == 0 ? kModeRefuse : kModeClaim, stamps};
+            ProbeKey s;
+            s.pending = false;
+            if (act) probe_start(s, key, e, mask, sl);
+            uint32_t claims = 0;
+            int32_t res;
+            uint32_t out, lslot;
+            warp_claim<false>(c, s, res, out, lslot, claims);
+            if (act) {
+                admit_write(e, res, out, result, slot_out, pos_out, status);
+                pend = false;
+            }
+            const uint32_t wc = __reduce_add_sync(kFull, claims);
+            if (lane == 0 && wc) atomicAdd_block(&s_claims, (unsigned long long)wc);
+            __syncthreads();
+            left -= s_claims;  // <= left: at most `left` entries claimed
+            admitted += s_claims;
+            __syncthreads();  // s_warp and s_claims are rewritten next round
+        }
+    }
+    if (threadIdx.x == 0 && admitted) atomicAdd(counter + 4, admitted);
+}
+
+// End of a claim kernel: the last CTA to finish (every CTA counts itself on
+// counter[5] after a fence) runs the admission pass when the call deferred
+// entries, and resets counter[5] for the next call.  Every CTA of the grid
+// must call it.
+__device__ __forceinline__ void admit_if_last(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
+                                              unsigned long long *counter, unsigned long long epoch,
+                                              unsigned long long *stamps, const uint8_t *keys, const uint32_t *slots,
+                                              uint64_t n, const int64_t *key_off, uint32_t R, int32_t *result,
+                                              uint32_t *slot_out, uint32_t *pos_out, int32_t *status) {
+    __shared__ int s_last;
+    __threadfence();  // this CTA's results and counts are visible to the GPU before it counts itself
+    __syncthreads();
+    if (threadIdx.x == 0) s_last = atomicAdd(counter + 5, 1ull) == (unsigned long long)gridDim.x - 1ull;
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    if (threadIdx.x == 0) counter[5] = 0;
+    if (__ldcg(counter + 2) == 0) return;  // nothing deferred: the claim kernel decided every entry
+    store_admit(table, mask, max_probe, capacity, counter, epoch, stamps, keys, slots, n, key_off, R, result,
+                slot_out, pos_out, status);
+}
+
 // List mode, or range mode for few long requests: one warp per 32
 // consecutive entries.
 __global__ void __launch_bounds__(256, 4)
@@ -686,6 +818,8 @@ k_store_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capac
     }
     pk::pdl_launch_dependents();
     count_claims(block_sums, claims, e < n && res == PK_STORE_DEFERRED, counter);
+    admit_if_last(table, mask, max_probe, capacity, counter, epoch, stamps, keys, slots, n, key_off, R, result, slot_out,
+                  slot_out, status);
 }
 
 // Range mode for many short requests: one warp per request, no search.
@@ -771,6 +905,8 @@ k_store_claim_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t c
     }
     pk::pdl_launch_dependents();
     count_claims(block_sums, claims, deferred, counter);
+    admit_if_last(table, mask, max_probe, capacity, counter, epoch, stamps, keys, slots, n, key_off, R, result, slot_out,
+                  slot_out, status);
 }
 
 // ---------------------------------------------------------------------------
@@ -910,6 +1046,8 @@ k_lookup_store_req(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t 
                              claims, deferred, true);
     }
     count_claims(block_sums, claims, deferred, counter);
+    admit_if_last(table, mask, max_probe, capacity, counter, epoch, stamps, keys, new_slots, key_capacity, key_off, R,
+                  result, slot_out, slot_out, status);
 }
 
 // Few long requests: one warp per 32 consecutive keys; k_lookup_store_tail
@@ -949,6 +1087,8 @@ k_lookup_store(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capa
     }
     pk::pdl_launch_dependents();
     count_claims(block_sums, claims, e < end && res == PK_STORE_DEFERRED, counter);
+    admit_if_last(table, mask, max_probe, capacity, counter, epoch, stamps, keys, new_slots, key_capacity, key_off, R,
+                  result, slot_out, slot_out, status);
 }
 
 // One warp per request: h_r = the first miss (slot PK_NO_SLOT), entries below
@@ -983,125 +1123,6 @@ k_lookup_store_tail(const int64_t *key_off, uint32_t R, uint64_t key_capacity,
     }
     if (lane == 0) hit[r] = (int32_t)h;
     if (arg) set_status(status, PK_ERR_ARG);
-}
-
-// Result of a deferred entry decided by the admit kernel.  pos_out: where a
-// PENDING entry's table position goes (slot_out for a context; the
-// allocation-free store keeps positions apart and writes PK_NO_SLOT to
-// slot_out).
-__device__ __forceinline__ void admit_write(uint64_t e, int32_t res, uint32_t out, int32_t *result,
-                                            uint32_t *slot_out, uint32_t *pos_out, int32_t *status) {
-    result[e] = res;
-    if (res == PK_STORE_PENDING && pos_out != slot_out) {
-        pos_out[e] = out;
-        slot_out[e] = PK_NO_SLOT;
-    } else {
-        slot_out[e] = out;
-    }
-    if (res < 0) set_status(status, res);
-}
-
-// Store, admit kernel (see the store comment above).  The call's entries are
-// [0, n), or [0, min(n, key_off[R])) in range and lookup-and-store mode;
-// counter[0] + counter[3] is the entry count after the claim kernel,
-// counter[2] the number of DEFERRED entries; keys claimed here are added to
-// counter[4].
-// Within the call the entry count can only reach capacity - 1: the claim
-// kernel claims only when the whole call fits, and here at most `room` keys
-// are claimed.
-__device__ __forceinline__ void store_admit(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity,
-                                            unsigned long long *counter, unsigned long long epoch,
-                                            unsigned long long *stamps, const uint8_t *keys, const uint32_t *slots,
-                                            uint64_t n, const int64_t *key_off, uint32_t R, int32_t *result,
-                                            uint32_t *slot_out, uint32_t *pos_out, int32_t *status) {
-    __shared__ uint32_t s_warp[8];
-    __shared__ unsigned long long s_claims;
-    const unsigned long long deferred = __ldcg(counter + 2);
-    if (deferred == 0) return;  // every key was decided by the claim kernel
-    const unsigned long long count = __ldcg(counter) + __ldcg(counter + 3);
-    const unsigned long long room = count + 1 < capacity ? capacity - 1 - count : 0ull;
-    uint64_t end = n;
-    if (key_off) {
-        const int64_t t = R ? __ldcg(key_off + R) : 0;
-        if (t < (int64_t)end) end = t > 0 ? (uint64_t)t : 0;
-    }
-    const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    if (deferred <= room) {
-        // At most `deferred` distinct keys: all fit.  Claimed in parallel.
-        const ClaimCtx c{table, mask, max_probe, epoch, kModeClaim, stamps};
-        uint32_t claims = 0;
-        if (threadIdx.x == 0) s_claims = 0;
-        __syncthreads();
-        for (uint64_t base = (uint64_t)blockIdx.x * blockDim.x + 32 * warp; base < end;
-             base += (uint64_t)gridDim.x * blockDim.x) {  // uniform per warp
-            const uint64_t e = base + lane;
-            ProbeKey s;
-            s.pending = false;
-            if (e < end && __ldcg(result + e) == PK_STORE_DEFERRED)
-                probe_start(s, ld_cg_v4(keys + 32 * e), e, mask, __ldcg(slots + e));
-            const bool mine = s.pending;
-            int32_t res;
-            uint32_t out, lslot;
-            warp_claim<false>(c, s, res, out, lslot, claims);
-            if (mine) admit_write(e, res, out, result, slot_out, pos_out, status);
-        }
-        const uint32_t wc = __reduce_add_sync(kFull, claims);
-        if (lane == 0 && wc) atomicAdd_block(&s_claims, (unsigned long long)wc);
-        __syncthreads();
-        if (threadIdx.x == 0 && s_claims) atomicAdd(counter + 4, s_claims);
-        return;
-    }
-    // More deferred entries than room: one CTA walks them in index order, 256
-    // at a time.  Each round the first `left` undecided entries of the tile
-    // (at most `left` distinct keys) claim or bid; once the room is gone the
-    // rest only bid on keys this call claimed, or are refused.  Every round
-    // decides at least one entry.
-    if (blockIdx.x != 0) return;
-    unsigned long long left = room, admitted = 0;
-    for (uint64_t base = 0; base < end; base += blockDim.x) {
-        const uint64_t e = base + threadIdx.x;
-        bool pend = e < end && __ldcg(result + e) == PK_STORE_DEFERRED;
-        const uint4 key = pend ? ld_cg_v4(keys + 32 * e) : make_uint4(0, 0, 0, 0);
-        const uint32_t sl = pend ? __ldcg(slots + e) : 0u;
-        for (;;) {
-            const uint32_t ball = __ballot_sync(kFull, pend);
-            if (lane == 0) s_warp[warp] = __popc(ball);
-            if (threadIdx.x == 0) s_claims = 0;
-            if (__syncthreads_count(pend) == 0) break;  // the tile is decided (uniform)
-            uint32_t rank = __popc(ball & lanemask_lt());
-            for (uint32_t w = 0; w < warp; ++w) rank += s_warp[w];
-            const bool act = pend && (left == 0 || rank < left);
-            const ClaimCtx c{table, mask, max_probe, epoch, left == 0 ? kModeRefuse : kModeClaim, stamps};
-            ProbeKey s;
-            s.pending = false;
-            if (act) probe_start(s, key, e, mask, sl);
-            uint32_t claims = 0;
-            int32_t res;
-            uint32_t out, lslot;
-            warp_claim<false>(c, s, res, out, lslot, claims);
-            if (act) {
-                admit_write(e, res, out, result, slot_out, pos_out, status);
-                pend = false;
-            }
-            const uint32_t wc = __reduce_add_sync(kFull, claims);
-            if (lane == 0 && wc) atomicAdd_block(&s_claims, (unsigned long long)wc);
-            __syncthreads();
-            left -= s_claims;  // <= left: at most `left` entries claimed
-            admitted += s_claims;
-            __syncthreads();  // s_warp and s_claims are rewritten next round
-        }
-    }
-    if (threadIdx.x == 0 && admitted) atomicAdd(counter + 4, admitted);
-}
-
-__global__ void __launch_bounds__(256)
-k_store_admit(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity, unsigned long long *counter,
-              unsigned long long epoch, unsigned long long *stamps, const uint8_t *keys, const uint32_t *slots,
-              uint64_t n, const int64_t *key_off, uint32_t R, int32_t *result, uint32_t *slot_out, int32_t *status) {
-    pk::pdl_launch_dependents();
-    pk::pdl_wait(table, counter, stamps, keys, slots, key_off, result, slot_out, status);
-    store_admit(table, mask, max_probe, capacity, counter, epoch, stamps, keys, slots, n, key_off, R, result,
-                slot_out, slot_out, status);
 }
 
 // Store, last kernel: each PENDING entry reads its key's slot/owner word,
@@ -1183,9 +1204,10 @@ __global__ void k_mark_loaded(pk_entry *table, uint64_t capacity) {
 struct NoallocScratch {
     // [0] entries in the table (set by the scan), [1] largest call number
     // found in the table, [2] entries deferred in this call, [3] keys its
-    // claim kernel claimed, [4] keys its admit kernel claimed: [0] and [2..4]
-    // are the words a context's counter holds at the same indices
-    unsigned long long word[5];
+    // claims claimed, [4] keys its admission pass claimed, [5] CTAs of the
+    // claim kernel done: [0] and [2..5] are the words a context's counter
+    // holds at the same indices
+    unsigned long long word[6];
     uint32_t pos[PK_NOALLOC_MAX_ENTRIES];  // table position of each PENDING entry
 };
 static __device__ __align__(256) NoallocScratch g_noalloc_scratch;
@@ -1253,17 +1275,8 @@ k_noalloc_claim(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t cap
         if (res < 0) set_status(status, res);
     }
     count_claims(block_sums, claims, e < n && res == PK_STORE_DEFERRED, sc->word);
-}
-
-// The admit kernel of the allocation-free store: the call number comes
-// from scratch, and PENDING positions go there.
-__global__ void __launch_bounds__(256)
-k_noalloc_admit(pk_entry *table, uint64_t mask, uint32_t max_probe, uint64_t capacity, NoallocScratch *sc,
-                const uint8_t *keys, const uint32_t *slots, uint64_t n, const int64_t *key_off, uint32_t R,
-                int32_t *result, uint32_t *slot_out, int32_t *status) {
-    const unsigned long long epoch = ld_volatile_u64(&sc->word[1]) + 1ull;
-    store_admit(table, mask, max_probe, capacity, sc->word, epoch, nullptr, keys, slots, n, key_off, R, result,
-                slot_out, sc->pos, status);
+    admit_if_last(table, mask, max_probe, capacity, sc->word, epoch, nullptr, keys, slots, n, key_off, R, result,
+                  slot_out, sc->pos, status);
 }
 
 __global__ void __launch_bounds__(256)
@@ -1277,14 +1290,6 @@ k_noalloc_finalize(const pk_entry *table, const NoallocScratch *sc, uint64_t n, 
 }
 
 unsigned grid_for(uint64_t n, unsigned block) { return (unsigned)((n + block - 1) / block); }
-
-// Grid of the admit kernel: grid-strided, at most two CTAs per SM (a launch
-// that usually finds nothing to do).
-unsigned admit_grid(uint64_t n, uint32_t sms) {
-    const unsigned g = grid_for(n, 256);
-    const unsigned cap = sms ? 2u * sms : g;
-    return g < cap ? g : (cap ? cap : 1u);
-}
 
 // Per-request kernels when the batch has many short requests; per-key kernels
 // when a few requests carry many keys each (a warp per request would then
@@ -1367,10 +1372,6 @@ cudaError_t pk_launch_store(const pk_ctx *ctx, unsigned long long epoch, const u
                       ctx->counter_dev, epoch, ctx->stamps, keys, slots, n, key_off, hit_chunks, R, result, slot_out, status);
     }
     if (e == cudaSuccess)
-        e = pk_launch(k_store_admit, admit_grid(n, ctx->sm_count), 256, s, ctx->table, mask, ctx->max_probe,
-                      ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, slots, n, key_off, R, result,
-                      slot_out, status);
-    if (e == cudaSuccess)
         e = pk_launch(k_store_finalize, grid_for(n, 256), 256, s, (const pk_entry *)ctx->table, n, key_off, R, result,
                       slot_out, ctx->counter_dev);
     return e != cudaSuccess ? e : cudaGetLastError();
@@ -1409,10 +1410,6 @@ cudaError_t pk_launch_lookup_store(const pk_ctx *ctx, unsigned long long epoch, 
             e = pk_launch(k_lookup_store_tail, grid_for(32ull * R, 256), 256, s, key_off, R, key_capacity,
                           (const uint32_t *)slots, hit_chunks, result, slot_out, status);
     }
-    if (e == cudaSuccess && key_capacity)
-        e = pk_launch(k_store_admit, admit_grid(key_capacity, ctx->sm_count), 256, s, ctx->table, mask,
-                      ctx->max_probe, ctx->capacity, ctx->counter_dev, epoch, ctx->stamps, keys, new_slots,
-                      key_capacity, key_off, R, result, slot_out, status);
     if (e == cudaSuccess && key_capacity)
         e = pk_launch(k_store_finalize, grid_for(key_capacity, 256), 256, s, (const pk_entry *)ctx->table,
                       key_capacity, key_off, R, result, slot_out, ctx->counter_dev);
@@ -1461,7 +1458,7 @@ cudaError_t pk_launch_store_noalloc(pk_entry *table, uint32_t capacity_log2, uin
     if (!sc) return cudaErrorInvalidSymbol;
     if (n == 0) return cudaSuccess;
     const uint64_t capacity = 1ull << capacity_log2;
-    // the five counter words must start at zero; pos needs no clearing
+    // the counter words must start at zero; pos needs no clearing
     e = cudaMemsetAsync(sc, 0, sizeof sc->word, s);
     if (e != cudaSuccess) return e;
     const uint64_t scan_blocks = (capacity + 255) / 256;
@@ -1471,8 +1468,6 @@ cudaError_t pk_launch_store_noalloc(pk_entry *table, uint32_t capacity_log2, uin
     k_noalloc_scan<<<(unsigned)(scan_blocks < scan_cap ? scan_blocks : scan_cap), 256, 0, s>>>(table, capacity, sc);
     k_noalloc_claim<<<grid_for(n, 256), 256, 0, s>>>(table, capacity - 1, max_probe, capacity, sc, keys, slots, n,
                                                       key_off, hit_chunks, Rm, result, slot_out, status);
-    k_noalloc_admit<<<admit_grid(n, sms), 256, 0, s>>>(table, capacity - 1, max_probe, capacity, sc, keys, slots, n,
-                                                        key_off, Rm, result, slot_out, status);
     k_noalloc_finalize<<<grid_for(n, 256), 256, 0, s>>>(table, sc, n, result, slot_out);
     return cudaGetLastError();
 }
