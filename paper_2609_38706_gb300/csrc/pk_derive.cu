@@ -339,17 +339,25 @@ k_chunk_digest(const int32_t *tokens, const int64_t *tok_off,
 //      (51 instead of 30 cycles per round, measured) while schedule warps
 //      share another; paired on one sub-partition, the schedule fills the
 //      issue slots the rounds warp's dependency chain leaves idle.  Block 1's
-//      schedule is published in one piece.  Named barriers of pair p:
-//      1 + 3p block-1 schedule; 2 + 3p block-2 schedule; 3 + 3p k_i published.
+//      schedule is published in two slices, t = 16..31 and 32..63 (the rounds
+//      warp waits for the burst of block-1 schedule work after each k_{i-1},
+//      so the smaller first slice lets its rounds 16..31 overlap the rest:
+//      small-block key derivation 654 -> 641 us; three slices: 646).  The
+//      first slice's barrier also marks block 2 of the step ready (written
+//      before it), which keeps the pairs within the 16 named barriers.  Named
+//      barriers of pair p: 1 + 3p block-1 slice 1 and block 2; 2 + 3p block-1
+//      slice 2; 3 + 3p k_i published.
 // Per pair both warps run the same number of steps (the lanes' maximum), so
 // every phase of every barrier gets exactly one arrive and one sync; the
 // schedule warp signals the block-2 barrier for step i only after it has
 // passed the k barrier of step i-1 (so after the rounds warp has synced the
-// block-2 barrier of step i-1), and the block-1 barrier of step i only after
-// the k barrier of step i-1 (after the rounds warp's block-1 sync of step
+// block-2 barrier of step i-1), and the block-1 barriers of step i only after
+// the k barrier of step i-1 (after the rounds warp's block-1 syncs of step
 // i-1): it never arrives twice on a barrier the rounds warp has not yet
-// synced.  Lanes past their own request's last chunk keep computing (masked)
-// so that the warps stay aligned.
+// synced.  Block 2's buffer for step i + 1 is written after the k barrier of
+// step i - 1, when the rounds warp has finished the block 2 that last used
+// it.  Lanes past their own request's last chunk keep computing (masked) so
+// that the warps stay aligned.
 // ---------------------------------------------------------------------------
 constexpr int kChainLanes = 32;
 
@@ -393,12 +401,21 @@ __device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint32_t (*kw)[
 // At most 64 registers (no spills): uncapped, the compiler took 81 and a small-block step whose
 // lookup-and-store launch overlaps the chain's tail ran 910 -> 955 us.  `groups` = ceil(R / 32); with
 // kPairs = 4, CTA c serves groups [c * groups / gridDim.x, (c + 1) * groups / gridDim.x), at most four.
-// FS: the form (pk_sha256.cuh) of the schedule warp's additions, `one` its run-time 1.  The rounds warp
-// keeps the compiler's form: its dependency chain sets the step time, and a multiply-add's longer latency
-// there made the four-pair chain slower (small-block key derivation 674 -> 718 us with every addition on the
-// FMA pipe).  With four pairs each sub-partition runs a rounds and a schedule warp on one ALU pipe, so the
-// schedule warp's additions go to the FMA pipe.
-template <int kPairs, int FS>
+// FS1, FS2: the forms (pk_sha256.cuh) of the schedule warp's additions for block 1 and block 2, `one` their
+// run-time 1 (with one pair per CTA the two blocks share one loop and FS1).  The rounds warp keeps the
+// compiler's form: its dependency chain sets the step time, and a multiply-add's longer latency there made
+// the four-pair chain slower (small-block key derivation 674 -> 718 us with every addition on the FMA pipe).
+// With four pairs each sub-partition runs a rounds warp and a schedule warp, whose two blocks differ:
+// block 1's schedule (k_{i-1} || d) can start only when k_{i-1} is published, and the rounds warp waits for
+// it after its 16th round, so it keeps the short-latency form; block 2's (c_i || padding) is made a step
+// ahead, off the critical path, and its additions go to the FMA pipe, where they do not compete with the
+// rounds warp's logic.  Small-block key derivation, measured: 683.7 us with both blocks in one loop and all
+// schedule additions on the FMA pipe; 674.8 with all on the ALU; 661.9 with the blocks in two loops, all on
+// the ALU; 655.8 as here.  Moving the small sigmas' shifts or rotations to the FMA pipe as well (mul.hi /
+// mad.lo by 2^(32-n): 4 and 6 cycles per warp instruction there) lost on either block (666-707 us): the
+// rounds warp's own multiply-adds queue behind them.  Block 2's first 16 words (K_t + W_t, set by
+// block2_head) and step 0's whole block 2, made before the loop, take FS1: 668 -> 654 us against FS2.
+template <int kPairs, int FS1, int FS2>
 __global__ void __launch_bounds__(2 * kChainLanes * kPairs, kPairs == 1 ? 15 : 4)
 k_chain(const int64_t *key_off, const uint32_t *desc_idx,
         const uint8_t *digests, uint32_t R, uint32_t D, uint8_t *keys, uint32_t groups, uint32_t one) {
@@ -418,7 +435,8 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
     }
     // named barriers of this pair (compile-time ids with one pair per CTA)
     const int bar_s1 = kPairs == 1 ? 1 : 1 + 3 * (int)pair;  // block-1 schedule (first slice)
-    const int bar_b2 = kPairs == 1 ? 4 : 2 + 3 * (int)pair;  // block-2 schedule
+    const int bar_s1b = kPairs == 1 ? 2 : 2 + 3 * (int)pair;  // block-1 schedule (second slice)
+    const int bar_b2 = kPairs == 1 ? 4 : -1;                  // block-2 schedule (four pairs: with bar_s1)
     const int bar_k = kPairs == 1 ? 5 : 3 + 3 * (int)pair;   // k_i published
     const uint32_t r = group * kChainLanes + lane;
     int64_t a = 0, n = 0;
@@ -452,11 +470,11 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
     uint4 *kq = reinterpret_cast<uint4 *>(keys + 32ull * a);
 
     if (sched) {  // ---------------- schedule warp ----------------
-        // The loop runs one copy of the 16-word schedule body for all six slices of a step (block-1
-        // slices 1-3 of step i, then block-2 slices 1-3 of step i+1).  The rounds warp on the next
-        // sub-partition slows down with the amount of distinct code this warp runs (per chain step,
-        // measured: 2206 ns with four unrolled copies, 2085 ns with one; 1950 ns with no schedule
-        // work at all).
+        // With one pair per CTA, one loop runs one copy of the 16-word schedule body for all six slices
+        // of a step (block-1 slices 1-3 of step i, then block-2 slices 1-3 of step i+1): the rounds warp
+        // on the next sub-partition slows down with the amount of distinct code this warp runs (per chain
+        // step, measured: 2206 ns with four unrolled copies, 2085 ns with one; 1950 ns with no schedule
+        // work at all).  With four pairs the two blocks have a loop each, in their own forms (FS1, FS2).
         // block 2 of step i: W = c_i (8 words) || 0x80000000, 0 x 6, 768; words 0..15 stored as K + W
         auto block2_head = [&](int64_t i, int buf, uint32_t w[16]) {
             if (i < n) {
@@ -472,15 +490,15 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
             for (int j = 9; j < 15; ++j) w[j] = 0;
             w[15] = 96u * 8u;
 #pragma unroll
-            for (int j = 0; j < 16; ++j) sm.kw2[buf][j][lane] = pk::add2<FS>(pk::kSha256K[j], w[j], one);
+            for (int j = 0; j < 16; ++j) sm.kw2[buf][j][lane] = pk::add2<FS1>(pk::kSha256K[j], w[j], one);
         };
         {
             uint32_t w[16];
             block2_head(0, 0, w);
 #pragma unroll 1
-            for (int q = 1; q < 4; ++q) schedule16<FS>(w, sm.kw2[0], q, lane, one);
+            for (int q = 1; q < 4; ++q) schedule16<FS1>(w, sm.kw2[0], q, lane, one);
         }
-        bar_arrive(bar_b2);
+        if (kPairs == 1) bar_arrive(bar_b2);
 #pragma unroll 1
         for (int64_t i = 0; i < nmax; ++i) {
             if (i + 1 == nmax) pk::pdl_launch_dependents();
@@ -492,22 +510,32 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
                 bar_sync(bar_k);  // k_{i-1} published; the rounds warp has finished step i-1
 #pragma unroll
                 for (int j = 0; j < 8; ++j) w[j] = sm.kpub[j][lane];
-                bar_arrive(bar_b2);  // block-2 schedule of step i (made during the previous iteration)
+                if (kPairs == 1) bar_arrive(bar_b2);  // block-2 schedule of step i (made in the previous iteration)
             }
 #pragma unroll
             for (int j = 0; j < 8; ++j) w[8 + j] = dw[j];
-            const int slices = i + 1 < nmax ? 6 : 3;
             const int buf = (int)((i + 1) & 1);
+            if (kPairs == 1) {
+                const int slices = i + 1 < nmax ? 6 : 3;
 #pragma unroll 1
-            for (int sl = 1; sl <= slices; ++sl) {
-                if (sl == 4) block2_head(i + 1, buf, w);
-                schedule16<FS>(w, sl <= 3 ? sm.kw1 : sm.kw2[buf], sl <= 3 ? sl : sl - 3, lane, one);
-                if (kPairs == 1) {  // constant barrier ids (a run-time id reserves all 16 named barriers)
+                for (int sl = 1; sl <= slices; ++sl) {
+                    if (sl == 4) block2_head(i + 1, buf, w);
+                    schedule16<FS1>(w, sl <= 3 ? sm.kw1 : sm.kw2[buf], sl <= 3 ? sl : sl - 3, lane, one);
+                    // constant barrier ids (a run-time id reserves all 16 named barriers)
                     if (sl == 1) bar_arrive(1);
                     else if (sl == 2) bar_arrive(2);
                     else if (sl == 3) bar_arrive(3);
-                } else if (sl == 3) {
-                    bar_arrive(bar_s1);
+                }
+            } else {
+                schedule16<FS1>(w, sm.kw1, 1, lane, one);
+                bar_arrive(bar_s1);  // also: block 2 of step i ready
+#pragma unroll 1
+                for (int sl = 2; sl <= 3; ++sl) schedule16<FS1>(w, sm.kw1, sl, lane, one);
+                bar_arrive(bar_s1b);
+                if (i + 1 < nmax) {
+                    block2_head(i + 1, buf, w);
+#pragma unroll 1
+                    for (int sl = 1; sl <= 3; ++sl) schedule16<FS2>(w, sm.kw2[buf], sl, lane, one);
                 }
             }
         }
@@ -542,12 +570,13 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
         } else {
             bar_sync(bar_s1);
             rounds16_kw<pk::kAddsPlain>(v, sm.kw1, 1, lane, one);
+            bar_sync(bar_s1b);
             rounds16_kw<pk::kAddsPlain>(v, sm.kw1, 2, lane, one);
             rounds16_kw<pk::kAddsPlain>(v, sm.kw1, 3, lane, one);
         }
         uint32_t st[8] = {PK_IV0 + v[0], PK_IV1 + v[1], PK_IV2 + v[2], PK_IV3 + v[3],
                           PK_IV4 + v[4], PK_IV5 + v[5], PK_IV6 + v[6], PK_IV7 + v[7]};
-        bar_sync(bar_b2);  // block-2 schedule of step i
+        if (kPairs == 1) bar_sync(bar_b2);  // block-2 schedule of step i
         const uint32_t (*kw2)[kChainLanes] = sm.kw2[i & 1];
 #pragma unroll
         for (int j = 0; j < 8; ++j) v[j] = st[j];
@@ -583,7 +612,7 @@ cudaError_t chain_packed_attr() {
     if (dev < 0 || dev >= 256) return cudaErrorInvalidDevice;
     std::lock_guard<std::mutex> lock(mu);
     if (!done[dev]) {
-        e = cudaFuncSetAttribute(k_chain<4, pk::kAddsFma>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(k_chain<4, pk::kAddsPlain, pk::kAddsFma>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)kChainPackedSmem);
         if (e != cudaSuccess) return e;
         done[dev] = true;
@@ -648,13 +677,13 @@ cudaError_t pk_launch_derive_enc(const pk_ctx *ctx, const int32_t *tokens, uint6
     // per SM, each pair on its own sub-partition) for more groups.
     const uint32_t groups = grid_for(R, kChainLanes);
     if (ctx->sm_count == 0 || groups <= ctx->sm_count) {
-        e = pk_launch_smem(k_chain<1, pk::kAddsPlain>, groups, 2 * kChainLanes, sizeof(ChainSmem), s,
+        e = pk_launch_smem(k_chain<1, pk::kAddsPlain, pk::kAddsPlain>, groups, 2 * kChainLanes, sizeof(ChainSmem), s,
                            (const int64_t *)key_off, desc_idx, (const uint8_t *)digests, R, D, keys, groups, one);
     } else {
         e = chain_packed_attr();
         const uint32_t grid = groups <= 4 * ctx->sm_count ? ctx->sm_count : grid_for(groups, 4);
         if (e == cudaSuccess)
-            e = pk_launch_smem(k_chain<4, pk::kAddsFma>, grid, 8 * kChainLanes, kChainPackedSmem, s,
+            e = pk_launch_smem(k_chain<4, pk::kAddsPlain, pk::kAddsFma>, grid, 8 * kChainLanes, kChainPackedSmem, s,
                                (const int64_t *)key_off, desc_idx, (const uint8_t *)digests, R, D, keys, groups, one);
     }
     if (e != cudaSuccess) return e;
