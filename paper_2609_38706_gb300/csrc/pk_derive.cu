@@ -309,7 +309,7 @@ k_chunk_digest(const int32_t *tokens, const int64_t *tok_off,
         const int64_t g = tile + threadIdx.x;
         const int64_t g0 = g - (threadIdx.x & 31);
         if (g0 >= g_end) break;  // whole warp past the end (uniform per warp)
-        const uint32_t r = pk::lane_request(key_off, R, g0, g_end, g);
+        const uint32_t r = pk::lane_request_guess(key_off, R, g0, g_end, g);
         if (g < g_end) digest_chunk<F>(tokens, tok_off, key_off, r, g, C, sK, sPad, ring, keys, one);
         __syncwarp();
     }

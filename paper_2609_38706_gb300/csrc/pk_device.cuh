@@ -59,6 +59,59 @@ __device__ __forceinline__ uint32_t lane_request(const int64_t *key_off, uint32_
     return find_request_in(key_off, r0, r1 + 1, g < total ? g : total - 1);
 }
 
+// Same result as lane_request with one search: r0 (the request of the warp's
+// first item) by warp_find_request, then one 32-wide load of key_off[r0+1 ..]
+// and a search over those 32 values by shuffles (non-decreasing key_off: r = r0
+// + the count of them <= g, one of 33 outcomes: 6 halvings).  A lane whose item
+// lies past those 32 requests (only after runs of empty requests) falls back to
+// find_request_in.
+__device__ __forceinline__ uint32_t lane_request_window(const int64_t *key_off, uint32_t R, int64_t g0,
+                                                        int64_t total, int64_t g) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t r0 = warp_find_request(key_off, R, g0);
+    const uint64_t p = (uint64_t)r0 + 1 + lane;
+    const int64_t v = p <= R ? __ldcg(key_off + p) : INT64_MAX;
+    const int64_t gg = g < total ? g : total - 1;
+    int lo = 0, hi = 32;  // the first j with key_off[r0 + 1 + j] > gg lies in [lo, hi] (32: none of the 32)
+#pragma unroll
+    for (int it = 0; it < 6; ++it) {
+        const int mid = (lo + hi) >> 1;
+        const int64_t vm = __shfl_sync(0xffffffffu, v, mid < 31 ? mid : 31);
+        if (lo < hi) {
+            if (vm <= gg) lo = mid + 1; else hi = mid;
+        }
+    }
+    if (lo < 32) return r0 + (uint32_t)lo;
+    return find_request_in(key_off, r0 + 32, R, gg);
+}
+
+// Same result again, for batches of about equal requests: a guess from the mean
+// request size, r_g = g0 * R / total, one 32-wide load of key_off[w0 ..] with
+// w0 = r_g - 8, and the same shuffle search; used when that window brackets
+// every lane's item, else lane_request_window.
+__device__ __forceinline__ uint32_t lane_request_guess(const int64_t *key_off, uint32_t R, int64_t g0,
+                                                       int64_t total, int64_t g) {
+    const uint32_t lane = threadIdx.x & 31;
+    const int64_t gg = g < total ? g : total - 1;
+    uint32_t rg = (uint32_t)((float)g0 / (float)total * (float)R);
+    rg = rg >= R ? R - 1 : rg;
+    const uint32_t w0 = rg > 8 ? rg - 8 : 0;
+    const uint64_t p = (uint64_t)w0 + lane;
+    const int64_t u = p <= R ? __ldcg(key_off + p) : INT64_MAX;
+    const int64_t u0 = __shfl_sync(0xffffffffu, u, 0);
+    int lo = 1, hi = 32;  // the first j >= 1 with key_off[w0 + j] > gg lies in [lo, hi] (32: none of the 31)
+#pragma unroll
+    for (int it = 0; it < 6; ++it) {
+        const int mid = (lo + hi) >> 1;
+        const int64_t vm = __shfl_sync(0xffffffffu, u, mid < 31 ? mid : 31);
+        if (lo < hi) {
+            if (vm <= gg) lo = mid + 1; else hi = mid;
+        }
+    }
+    if (__all_sync(0xffffffffu, u0 <= g0 && lo < 32)) return w0 + (uint32_t)lo - 1;
+    return lane_request_window(key_off, R, g0, total, g);
+}
+
 }  // namespace pk
 
 namespace pk {

@@ -249,3 +249,31 @@ def test_many_requests_span_scan_tiles_and_parts(R, C):
     ko, keys, rko, rkeys = derive_both(kt, rows, rng.integers(0, 3, R), descs, C)
     assert np.array_equal(ko, rko) and np.array_equal(keys, rkeys)
     kt.close()
+
+
+@pytest.mark.parametrize("layout", ["uniform", "skewed", "empty_runs"])
+def test_chunk_to_request_mapping_paths(layout):
+    """The chunk-digest warps map their 32 chunks to requests from a guess
+    (requests of about equal size), checked against 32 loaded offsets, and fall
+    back to a search when the guess misses or the window ends inside a run of
+    empty requests.  Uniform requests take the guess; a skewed batch (a few
+    huge requests among small ones) misses it; runs of 40-200 empty requests
+    between short ones end the window early.  Keys compared with the oracle."""
+    rng = np.random.default_rng({"uniform": 1, "skewed": 2, "empty_runs": 3}[layout])
+    C = 16
+    if layout == "uniform":
+        lens = np.full(3000, 8 * C, np.int64)
+    elif layout == "skewed":
+        lens = rng.integers(0, 3 * C, 3000)
+        lens[rng.integers(0, 3000, 12)] = rng.integers(200 * C, 400 * C, 12)
+    else:
+        lens = np.zeros(6000, np.int64)
+        i = 0
+        while i < lens.size:
+            lens[i] = rng.integers(1, 6 * C)
+            i += 1 + int(rng.integers(40, 200)) if rng.random() < 0.3 else 1
+    rows = [rng.integers(0, 152064, int(n)).astype(np.int32) for n in lens]
+    kt = KT(C, log2=10)
+    ko, keys, rko, rkeys = derive_both(kt, rows, rng.integers(0, 2, lens.size), [DESC, dict(DESC, salt="m")], C)
+    assert np.array_equal(ko, rko) and np.array_equal(keys, rkeys)
+    kt.close()
