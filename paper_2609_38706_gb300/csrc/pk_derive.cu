@@ -86,7 +86,21 @@ k_chunk_offsets(const int64_t *tok_off, uint32_t R, uint64_t n_tokens, uint32_t 
     if (tid == 0) key_off[0] = 0;
     bool bad = false;
     long long carry = 0;
-    for (uint64_t base = 0; base < R; base += (uint64_t)kScanThreads * kScanItems) {
+    // a tile's inputs (its threads' tok_off[r0 .. r0 + kScanItems], desc_idx[r0 .. r0 + kScanItems)) are loaded
+    // one tile ahead, so that they are in flight during the previous tile's scan
+    constexpr uint64_t kTile = (uint64_t)kScanThreads * kScanItems;
+    int64_t to_cur[kScanItems + 1], to_nxt[kScanItems + 1] = {};
+    uint32_t di_cur[kScanItems], di_nxt[kScanItems] = {};
+    auto load_tile = [&](uint64_t base, int64_t *to, uint32_t *di) {
+        const uint64_t r0 = base + (uint64_t)tid * kScanItems;
+#pragma unroll
+        for (int j = 0; j <= kScanItems; ++j) to[j] = r0 + j <= R ? tok_off[r0 + j] : 0;
+#pragma unroll
+        for (int j = 0; j < kScanItems; ++j) di[j] = r0 + j < R ? desc_idx[r0 + j] : 0u;
+    };
+    if (R > 0) load_tile(0, to_cur, di_cur);
+    for (uint64_t base = 0; base < R; base += kTile) {
+        if (base + kTile < R) load_tile(base + kTile, to_nxt, di_nxt);
         const uint64_t r0 = base + (uint64_t)tid * kScanItems;
         long long n[kScanItems];
         long long local = 0;
@@ -95,8 +109,8 @@ k_chunk_offsets(const int64_t *tok_off, uint32_t R, uint64_t n_tokens, uint32_t 
             const uint64_t r = r0 + j;
             n[j] = 0;
             if (r < R) {
-                const int64_t a = tok_off[r], b = tok_off[r + 1];
-                if (a < 0 || b < a || (uint64_t)b > n_tokens || desc_idx[r] >= D) {
+                const int64_t a = to_cur[j], b = to_cur[j + 1];
+                if (a < 0 || b < a || (uint64_t)b > n_tokens || di_cur[j] >= D) {
                     bad = true;
                 } else {  // 32-bit division when the request fits (64-bit division is a long library sequence)
                     const uint64_t len = (uint64_t)(b - a);
@@ -136,6 +150,10 @@ k_chunk_offsets(const int64_t *tok_off, uint32_t R, uint64_t n_tokens, uint32_t 
         }
         carry += tile_total;
         __syncthreads();  // warp_sums and tile_total are reused by the next tile
+#pragma unroll
+        for (int j = 0; j <= kScanItems; ++j) to_cur[j] = to_nxt[j];
+#pragma unroll
+        for (int j = 0; j < kScanItems; ++j) di_cur[j] = di_nxt[j];
     }
     bad = __syncthreads_or(bad);
     if (bad || (unsigned long long)carry > key_capacity) {
@@ -206,7 +224,18 @@ __device__ __forceinline__ void digest_chunk(const int32_t *tokens, const int64_
     pk::init_state(st);
     const uint32_t nfull = C / 16;
     uint32_t w[16];
-    if (aligned) {
+    if (aligned && nfull == 1) {  // one data block: straight into registers
+        const uint4 *q = reinterpret_cast<const uint4 *>(src);
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const uint4 x = __ldcg(q + v);
+            w[4 * v + 0] = pk::bswap32(x.x);
+            w[4 * v + 1] = pk::bswap32(x.y);
+            w[4 * v + 2] = pk::bswap32(x.z);
+            w[4 * v + 3] = pk::bswap32(x.w);
+        }
+        pk::compress_rolled<F>(st, w, sK, one);
+    } else if (aligned) {
 #pragma unroll
         for (int b = 0; b < kStages - 1; ++b) {
             if ((uint32_t)b < nfull) cp_async_block(ring[b][threadIdx.x], src + 16 * b);
