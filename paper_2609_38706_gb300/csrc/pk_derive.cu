@@ -224,18 +224,7 @@ __device__ __forceinline__ void digest_chunk(const int32_t *tokens, const int64_
     pk::init_state(st);
     const uint32_t nfull = C / 16;
     uint32_t w[16];
-    if (aligned && nfull == 1) {  // one data block: straight into registers
-        const uint4 *q = reinterpret_cast<const uint4 *>(src);
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-            const uint4 x = __ldcg(q + v);
-            w[4 * v + 0] = pk::bswap32(x.x);
-            w[4 * v + 1] = pk::bswap32(x.y);
-            w[4 * v + 2] = pk::bswap32(x.z);
-            w[4 * v + 3] = pk::bswap32(x.w);
-        }
-        pk::compress_rolled<F>(st, w, sK, one);
-    } else if (aligned) {
+    if (aligned) {
 #pragma unroll
         for (int b = 0; b < kStages - 1; ++b) {
             if ((uint32_t)b < nfull) cp_async_block(ring[b][threadIdx.x], src + 16 * b);
