@@ -382,21 +382,25 @@ constexpr int kChainLanes = 32;
 __device__ __forceinline__ void bar_sync(int id) { asm volatile("bar.sync %0, 64;" ::"r"(id) : "memory"); }
 __device__ __forceinline__ void bar_arrive(int id) { asm volatile("bar.arrive %0, 64;" ::"r"(id) : "memory"); }
 
+// K+W words pass between the two warps four to a 16-byte vector ([t / 4][lane]): one shared-memory
+// instruction per four words on either side.
 struct ChainSmem {
-    uint32_t kw1[64][kChainLanes];     // block-1 K+W, t = 16..63 used
-    uint32_t kw2[2][64][kChainLanes];  // block-2 K+W, double-buffered by step parity
-    uint32_t kpub[8][kChainLanes];     // k_{i-1} for the schedule warp
+    uint4 kw1[16][kChainLanes];     // block-1 K+W, t = 16..63 used
+    uint4 kw2[2][16][kChainLanes];  // block-2 K+W, double-buffered by step parity
+    uint4 kpub[2][kChainLanes];     // k_{i-1} for the schedule warp
 };
 
-// 16 schedule words t = 16q .. 16q+15 of the ring w (in place), K_t + W_t -> out[t][lane]
+// 16 schedule words t = 16q .. 16q+15 of the ring w (in place), K_t + W_t -> out[t / 4][lane]
 // (F: round form of pk_sha256.cuh, `one` its run-time 1)
 template <int F>
-__device__ __forceinline__ void schedule16(uint32_t w[16], uint32_t (*out)[kChainLanes], int q, uint32_t lane,
+__device__ __forceinline__ void schedule16(uint32_t w[16], uint4 (*out)[kChainLanes], int q, uint32_t lane,
                                            uint32_t one) {
+    uint32_t o[4];
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
         pk::sched_word<F>(w, j, one);
-        out[16 * q + j][lane] = pk::add2<F>(pk::kSha256K[16 * q + j], w[j], one);
+        o[j & 3] = pk::add2<F>(pk::kSha256K[16 * q + j], w[j], one);
+        if ((j & 3) == 3) out[4 * q + (j >> 2)][lane] = make_uint4(o[0], o[1], o[2], o[3]);
     }
 }
 
@@ -405,12 +409,18 @@ __device__ __forceinline__ void schedule16(uint32_t w[16], uint32_t (*out)[kChai
 // runs 64 rounds in 2018 instead of 2241 cycles when no round waits on its
 // shared-memory read)
 template <int F>
-__device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint32_t (*kw)[kChainLanes], int q, uint32_t lane,
+__device__ __forceinline__ void rounds16_kw(uint32_t v[8], const uint4 (*kw)[kChainLanes], int q, uint32_t lane,
                                             uint32_t one) {
     uint32_t a = v[0], b = v[1], c = v[2], d = v[3], e = v[4], f = v[5], g = v[6], h = v[7];
     uint32_t x[16];
 #pragma unroll
-    for (int j = 0; j < 16; ++j) x[j] = kw[16 * q + j][lane];
+    for (int m = 0; m < 4; ++m) {
+        const uint4 y = kw[4 * q + m][lane];
+        x[4 * m] = y.x;
+        x[4 * m + 1] = y.y;
+        x[4 * m + 2] = y.z;
+        x[4 * m + 3] = y.w;
+    }
 #pragma unroll
     for (int j = 0; j < 16; ++j) pk::round_kw<F>(a, b, c, d, e, f, g, h, x[j], one);
     v[0] = a; v[1] = b; v[2] = c; v[3] = d; v[4] = e; v[5] = f; v[6] = g; v[7] = h;
@@ -508,7 +518,11 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
             for (int j = 9; j < 15; ++j) w[j] = 0;
             w[15] = 96u * 8u;
 #pragma unroll
-            for (int j = 0; j < 16; ++j) sm.kw2[buf][j][lane] = pk::add2<FS1>(pk::kSha256K[j], w[j], one);
+            for (int m = 0; m < 4; ++m)
+                sm.kw2[buf][m][lane] = make_uint4(
+                    pk::add2<FS1>(pk::kSha256K[4 * m], w[4 * m], one), pk::add2<FS1>(pk::kSha256K[4 * m + 1], w[4 * m + 1], one),
+                    pk::add2<FS1>(pk::kSha256K[4 * m + 2], w[4 * m + 2], one),
+                    pk::add2<FS1>(pk::kSha256K[4 * m + 3], w[4 * m + 3], one));
         };
         {
             uint32_t w[16];
@@ -527,7 +541,13 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
             } else {
                 bar_sync(bar_k);  // k_{i-1} published; the rounds warp has finished step i-1
 #pragma unroll
-                for (int j = 0; j < 8; ++j) w[j] = sm.kpub[j][lane];
+                for (int m = 0; m < 2; ++m) {
+                    const uint4 y = sm.kpub[m][lane];
+                    w[4 * m] = y.x;
+                    w[4 * m + 1] = y.y;
+                    w[4 * m + 2] = y.z;
+                    w[4 * m + 3] = y.w;
+                }
                 if (kPairs == 1) bar_arrive(bar_b2);  // block-2 schedule of step i (made in the previous iteration)
             }
 #pragma unroll
@@ -595,7 +615,7 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
         uint32_t st[8] = {PK_IV0 + v[0], PK_IV1 + v[1], PK_IV2 + v[2], PK_IV3 + v[3],
                           PK_IV4 + v[4], PK_IV5 + v[5], PK_IV6 + v[6], PK_IV7 + v[7]};
         if (kPairs == 1) bar_sync(bar_b2);  // block-2 schedule of step i
-        const uint32_t (*kw2)[kChainLanes] = sm.kw2[i & 1];
+        const uint4 (*kw2)[kChainLanes] = sm.kw2[i & 1];
 #pragma unroll
         for (int j = 0; j < 8; ++j) v[j] = st[j];
 #pragma unroll 1
@@ -605,7 +625,7 @@ k_chain(const int64_t *key_off, const uint32_t *desc_idx,
         if (i < n) store_digest(keys + 32ull * (a + i), p);
         if (i + 1 < nmax) {
 #pragma unroll
-            for (int j = 0; j < 8; ++j) sm.kpub[j][lane] = p[j];
+            for (int m = 0; m < 2; ++m) sm.kpub[m][lane] = make_uint4(p[4 * m], p[4 * m + 1], p[4 * m + 2], p[4 * m + 3]);
             bar_arrive(bar_k);
         }
     }
