@@ -27,6 +27,7 @@ the device-to-host copy of the results.
 from __future__ import annotations
 
 import argparse
+import gc
 import json
 import os
 import statistics
@@ -415,7 +416,10 @@ def main():
         kt.load(snapshot)
         flush.fill_(1)
 
-    spin_cycles = int(300e-6 * 2.0e9)
+    # The spin kernel ahead of each step (outside its events) keeps the device busy while the host enqueues
+    # the step: about 1 ms, so that a short host pause inside the enqueue (a driver query of the clock
+    # sampler, say) does not leave the device idle between the step's events.
+    spin_cycles = int(1e-3 * 2.0e9)
     n_keys = wl.n_keys()
 
     # ---- warm-up, then timed device-resident steps ----
@@ -441,6 +445,8 @@ def main():
     # Only a start and an end event per timed step: an event recorded between two kernels also ends the
     # programmatic overlap of the second with the first.
     step_ms = []
+    gc.collect()
+    gc.disable()  # no collection pause while a step is being enqueued
     for _ in range(args.steps):
         between_steps()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -450,6 +456,7 @@ def main():
         e1.record(stream)
         torch.cuda.synchronize()
         step_ms.append(e0.elapsed_time(e1))
+    gc.enable()
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
